@@ -1,0 +1,25 @@
+"""Oracle for the SEED draft/verify attention path -- TEST INFRASTRUCTURE ONLY.
+
+A plain, slow, float64 CPU statement of what the path computes, written from
+the paper (SEED: Self-Speculative Decoding via Implicit Encoder-Decoder):
+
+* ``attention``  -- softmax attention over the KV cache (Sec. 4.1, "Cheap
+  drafting between verifications": the drafter's cross-attention is ordinary
+  self-attention over the cache), for the draft query and for the k+1 causal
+  verify queries (Alg. 2, drafting and verification phases).
+* ``cache``      -- the paged KV cache: slot of a logical position, gathering a
+  sequence's rows, appending rows (Alg. 2; cache updates left implicit in
+  Sec. 3).
+* ``accept``     -- greedy longest-prefix acceptance, bonus token and the
+  commit/rollback of cache rows (Alg. 2, acceptance and truncation steps).
+* ``toy_model``  -- a tiny float64 transformer running Alg. 2 end to end and
+  plain greedy decoding, for the exactness property of Sec. 4.1.
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and the ``cpu_baseline`` /
+``--impl reference`` legs of ``bench.py`` may import this package.  It shares
+no code with the CUDA path and never imports it.
+
+Parity status: every function here is pinned by ``tests/test_oracle_*.py``
+(brute force, closed forms, library cross-checks, invariants, exactness of the
+end-to-end loop).  Nothing is "parity unpinned".
+"""
