@@ -1,0 +1,197 @@
+/*
+ * seed.h -- C ABI of the SEED draft/verify attention path for NVIDIA GB300
+ * (sm_103a).
+ *
+ * SEED (Self-Speculative Decoding via Implicit Encoder-Decoder) drafts tokens
+ * with the last decoder layers of the model, fed raw token embeddings and
+ * attending to the deep KV cache the previous verification left behind
+ * (Sec. 4.1), then verifies d drafts with one (d+1)-token pass of the full
+ * model and keeps the greedy longest matching prefix plus a bonus token
+ * (Alg. 2).  This library implements the memory-bound steps of that loop:
+ *
+ *   seed_draft_kv_append / seed_draft_attn   -- one draft step, per decoder layer
+ *   seed_kv_append       / seed_verify_attn  -- the verify pass, per layer
+ *   seed_accept_commit                       -- acceptance and cache commit
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ * - All tensor pointers are DEVICE pointers, row-major, densely packed, owned
+ *   by the caller; the library never allocates, frees or synchronises, and
+ *   keeps no state between calls.  Calls are asynchronous on `stream` (a
+ *   cudaStream_t; NULL is the legacy default stream) and are safe to call
+ *   from several host threads on different streams.
+ * - bf16 tensors hold IEEE bfloat16 bit patterns; f32 outputs are IEEE float.
+ * - Host-side checks (null pointers, unsupported shapes, a too-small
+ *   workspace) return a status synchronously and launch nothing.
+ * - Data-dependent checks run on the device: a violation ORs a SEED_DEVERR_*
+ *   bit into *err_flag (an int32 in device memory, which the caller zeroes and
+ *   reads) and the offending work is skipped.  No kernel ever traps; outputs
+ *   of a call that raised a device error are unspecified, but no memory
+ *   outside the arguments is touched.
+ * - KV cache of one layer (a "paged" cache): K and V are each
+ *   [num_pages, hkv, page_size, head_dim] bf16.  Logical position `pos` of
+ *   sequence b lives in page page_table[b * max_pages + pos / page_size] at
+ *   offset pos % page_size.  A contiguous cache is the identity page order.
+ * - GQA: query head h reads KV head h / (hq / hkv).
+ * - Attention outputs are f32; lse is the natural-log sum of exp(scores).
+ */
+#ifndef SEED_H_
+#define SEED_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define SEED_ABI_VERSION 1
+#define SEED_MAX_KMAX 16        /* largest supported draft length d */
+
+typedef enum {
+  SEED_OK = 0,
+  SEED_ERR_NULL = 1,          /* a required pointer is NULL                    */
+  SEED_ERR_SHAPE = 2,         /* batch < 0, hq % hkv != 0, kmax out of range   */
+  SEED_ERR_RANGE = 3,         /* max_pages / num_pages out of range            */
+  SEED_ERR_UNSUPPORTED = 4,   /* head_dim, group size or page_size not built   */
+  SEED_ERR_CUDA = 5,          /* a CUDA runtime call failed (launch error)     */
+  SEED_ERR_WORKSPACE = 6      /* workspace too small or misaligned             */
+} seed_status_t;
+
+/* Device error bits (OR-ed into *err_flag). */
+#define SEED_DEVERR_CTX_LEN   1   /* ctx_len < 0, or rows past max_pages*page_size */
+#define SEED_DEVERR_DRAFT_LEN 2   /* draft_len outside [0, kmax]                    */
+#define SEED_DEVERR_NQ        4   /* n_q / n_new outside [0, kmax+1]                */
+#define SEED_DEVERR_PAGE      8   /* page id outside [0, num_pages)                 */
+#define SEED_DEVERR_KB        16  /* k_b outside [0, kmax]                          */
+#define SEED_DEVERR_WORKSPACE 32  /* more work units than the workspace holds       */
+#define SEED_DEVERR_TIMEOUT   64  /* a bounded on-chip wait gave up (never expected) */
+
+/* Shapes of one model's attention.  Supported: head_dim in {64, 128};
+ * hq / hkv in {1, 2, 4, 8}; page_size == 16; 1 <= kmax <= SEED_MAX_KMAX.
+ * scale == 0 selects 1/sqrt(head_dim) (the paper leaves the softmax scale to
+ * the base model; this is the usual one). */
+typedef struct {
+  int32_t hq;
+  int32_t hkv;
+  int32_t head_dim;
+  int32_t page_size;
+  int32_t kmax;
+  float scale;
+} seed_cfg_t;
+
+/* One layer's paged KV cache.  k, v: bf16 [num_pages, hkv, page_size,
+ * head_dim] (written only by the *_append calls); page_table: int32
+ * [batch, max_pages]. */
+typedef struct {
+  void* k;
+  void* v;
+  const int32_t* page_table;
+  int32_t max_pages;
+  int32_t num_pages;
+} seed_kv_t;
+
+int32_t seed_abi_version(void);
+const char* seed_status_string(seed_status_t status);
+
+/* Bytes of device workspace that seed_draft_attn and seed_verify_attn need
+ * for `batch` sequences with this cfg (independent of lengths).  The
+ * workspace must be 256-byte aligned and ZERO-FILLED before its first use;
+ * every call leaves it zero-filled again (it holds split partials and
+ * per-(sequence, KV head) arrival counters).  Returns 0 for an invalid cfg. */
+size_t seed_workspace_bytes(const seed_cfg_t* cfg, int32_t batch);
+
+/* Draft step, cache side (Alg. 2, drafting phase; Sec. 4.1 "Cheap drafting"):
+ * store the K/V row the drafter computed for X_draft[i-1] in one decoder layer
+ * as row i-1 of that layer's draft scratch.
+ *   k_new, v_new   bf16 [batch, hkv, head_dim]
+ *   draft_lens     int32 [batch]: i, the number of draft rows after this
+ *                  append (1..kmax); 0 skips the sequence
+ *   draft_k/v      bf16 [batch, hkv, kmax, head_dim], written at row i-1
+ * Device errors: SEED_DEVERR_DRAFT_LEN. */
+seed_status_t seed_draft_kv_append(const seed_cfg_t* cfg, int32_t batch,
+                                   const void* k_new, const void* v_new,
+                                   const int32_t* draft_lens,
+                                   void* draft_k, void* draft_v,
+                                   int32_t* err_flag, void* stream);
+
+/* Draft attention (Sec. 4.1 eq. for X_{n+1} from f_dec(H^0_n, KV^dec_{<n});
+ * Alg. 2 drafting phase): for each sequence b and query head h, softmax
+ * attention of q[b, h] over the ctx_lens[b] committed rows of this decoder
+ * layer's cache (the deep KV the last verification wrote) followed by the
+ * draft_lens[b] rows of the draft scratch (X_draft[0..i-1], the query's own
+ * row included).
+ *   q            bf16 [batch, hq, head_dim]
+ *   ctx_kv       this layer's cache (read only)
+ *   draft_k/v    bf16 [batch, hkv, kmax, head_dim]
+ *   ctx_lens     int32 [batch] >= 0
+ *   draft_lens   int32 [batch] in [0, kmax]; 0 skips the sequence (its out
+ *                and lse rows are left untouched)
+ *   out          f32 [batch, hq, head_dim]
+ *   lse          f32 [batch, hq], or NULL
+ *   ws           workspace of ws_bytes >= seed_workspace_bytes(cfg, batch)
+ * Device errors: SEED_DEVERR_CTX_LEN, _DRAFT_LEN, _PAGE, _WORKSPACE. */
+seed_status_t seed_draft_attn(const seed_cfg_t* cfg, int32_t batch, const void* q,
+                              seed_kv_t ctx_kv, const void* draft_k, const void* draft_v,
+                              const int32_t* ctx_lens, const int32_t* draft_lens,
+                              float* out, float* lse, void* ws, size_t ws_bytes,
+                              int32_t* err_flag, void* stream);
+
+/* Verify pass, cache side (Alg. 2 verification phase; Sec. 4.1 "Verification
+ * already does the encoder's work"): write the n_new[b] K/V rows the verifier
+ * computed for X_draft[0..n_new-1] at logical positions ctx_lens[b] ..
+ * ctx_lens[b] + n_new[b] - 1 of this layer's cache.
+ *   k_new, v_new  bf16 [batch, kmax+1, hkv, head_dim]
+ *   n_new         int32 [batch] in [0, kmax+1]
+ *   ctx_lens      int32 [batch] (not modified)
+ * Device errors: SEED_DEVERR_CTX_LEN, _NQ, _PAGE. */
+seed_status_t seed_kv_append(const seed_cfg_t* cfg, int32_t batch, seed_kv_t kv,
+                             const void* k_new, const void* v_new, const int32_t* n_new,
+                             const int32_t* ctx_lens, int32_t* err_flag, void* stream);
+
+/* Verify attention (Alg. 2 verification phase: (f_dec o f_enc) over
+ * X_draft[0..d] with the cache KV_{1..t-1}): query j of sequence b (token
+ * X_draft[j], j < n_q[b]) attends to rows 0 .. ctx_lens[b] + j of this
+ * layer's cache, which already holds the n_q[b] new rows (seed_kv_append):
+ * causal among the new rows, all committed rows visible.
+ *   q         bf16 [batch, kmax+1, hq, head_dim]
+ *   n_q       int32 [batch] in [0, kmax+1] (k_b + 1; 0 skips the sequence)
+ *   kv        this layer's cache (read only)
+ *   ctx_lens  int32 [batch]: committed rows before the new ones
+ *   out       f32 [batch, kmax+1, hq, head_dim] (rows j >= n_q untouched)
+ *   lse       f32 [batch, kmax+1, hq], or NULL
+ * Device errors: SEED_DEVERR_CTX_LEN, _NQ, _PAGE, _WORKSPACE. */
+seed_status_t seed_verify_attn(const seed_cfg_t* cfg, int32_t batch, const void* q,
+                               const int32_t* n_q, seed_kv_t kv, const int32_t* ctx_lens,
+                               float* out, float* lse, void* ws, size_t ws_bytes,
+                               int32_t* err_flag, void* stream);
+
+/* Greedy acceptance and cache commit/rollback (Alg. 2, after verification):
+ * n_b = number of leading i < k_b[b] with draft_ids[b,i] == target_ids[b,i];
+ * tokens[b] = draft_ids[b, 0..n_b-1] then the bonus target_ids[b, n_b];
+ * the rows of X_draft[0..n_b] (positions ctx_lens[b] .. ctx_lens[b]+n_b) are
+ * committed and their physical slots (page * page_size + offset) reported;
+ * rows past them are rolled back (left in place, never read again);
+ * ctx_lens[b] += n_b + 1.
+ *   draft_ids        int32 [batch, kmax]   (X_draft[1..kmax])
+ *   target_ids       int32 [batch, kmax+1] (argmax p_1..p_{kmax+1})
+ *   k_b              int32 [batch] in [0, kmax]
+ *   page_table       int32 [batch, max_pages]
+ *   ctx_lens         int32 [batch], updated in place
+ *   accepted         int32 [batch]: n_b
+ *   tokens           int32 [batch, kmax+1], -1 past n_b
+ *   committed_slots  int32 [batch, kmax+1], -1 past n_b
+ * Device errors: SEED_DEVERR_KB, _CTX_LEN (committed rows past capacity);
+ * the sequence is then left unchanged. */
+seed_status_t seed_accept_commit(int32_t batch, int32_t kmax, const int32_t* draft_ids,
+                                 const int32_t* target_ids, const int32_t* k_b,
+                                 const int32_t* page_table, int32_t max_pages,
+                                 int32_t page_size, int32_t* ctx_lens, int32_t* accepted,
+                                 int32_t* tokens, int32_t* committed_slots,
+                                 int32_t* err_flag, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SEED_H_ */

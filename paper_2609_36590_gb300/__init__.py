@@ -1,0 +1,244 @@
+"""Python binding of the SEED draft/verify attention library (include/seed.h).
+
+Argument marshalling only: every call checks that its torch tensors have the
+dtype, device, shape and layout the C ABI expects, passes their data pointers
+and the current CUDA stream to ``libseed.so``, and raises on a non-OK status.
+All arithmetic runs in the library's CUDA kernels; there is no fallback, and
+every entry point fails loudly when the library has not been built.
+
+Entry points carry the C names: seed_workspace_bytes, seed_draft_kv_append,
+seed_draft_attn, seed_kv_append, seed_verify_attn, seed_accept_commit.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libseed.so")
+
+SEED_OK = 0
+DEVERR = {1: "ctx_len", 2: "draft_len", 4: "n_q", 8: "page", 16: "k_b", 32: "workspace",
+          64: "timeout"}
+MAX_KMAX = 16
+
+
+class _Cfg(ctypes.Structure):
+    _fields_ = [("hq", ctypes.c_int32), ("hkv", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+                ("page_size", ctypes.c_int32), ("kmax", ctypes.c_int32), ("scale", ctypes.c_float)]
+
+
+class _KV(ctypes.Structure):
+    _fields_ = [("k", ctypes.c_void_p), ("v", ctypes.c_void_p), ("page_table", ctypes.c_void_p),
+                ("max_pages", ctypes.c_int32), ("num_pages", ctypes.c_int32)]
+
+
+_P = ctypes.c_void_p
+_I = ctypes.c_int32
+_SIGS = {
+    "seed_abi_version": (_I, []),
+    "seed_status_string": (ctypes.c_char_p, [_I]),
+    "seed_workspace_bytes": (ctypes.c_size_t, [ctypes.POINTER(_Cfg), _I]),
+    "seed_draft_kv_append": (_I, [ctypes.POINTER(_Cfg), _I, _P, _P, _P, _P, _P, _P, _P]),
+    "seed_draft_attn": (_I, [ctypes.POINTER(_Cfg), _I, _P, _KV, _P, _P, _P, _P, _P, _P, _P,
+                             ctypes.c_size_t, _P, _P]),
+    "seed_kv_append": (_I, [ctypes.POINTER(_Cfg), _I, _KV, _P, _P, _P, _P, _P, _P]),
+    "seed_verify_attn": (_I, [ctypes.POINTER(_Cfg), _I, _P, _P, _KV, _P, _P, _P, _P,
+                              ctypes.c_size_t, _P, _P]),
+    "seed_accept_commit": (_I, [_I, _I, _P, _P, _P, _P, _I, _I, _P, _P, _P, _P, _P, _P]),
+}
+
+
+def _load() -> ctypes.CDLL:
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(
+            f"{LIB_PATH} is missing: build it with `python -m paper_2609_36590_gb300.build` "
+            "(the SEED path has no CPU fallback)")
+    lib = ctypes.CDLL(LIB_PATH)
+    for name, (res, args) in _SIGS.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    return lib
+
+
+class _Lazy:
+    """Loads libseed.so on first use, so that the build script can import the
+    package before the library exists; every entry point fails loudly if it is
+    still missing then."""
+
+    _cdll = None
+
+    def __getattr__(self, name):
+        if _Lazy._cdll is None:
+            _Lazy._cdll = _load()
+        return getattr(_Lazy._cdll, name)
+
+
+_lib = _Lazy()
+
+
+class SeedError(RuntimeError):
+    pass
+
+
+def _check(status: int) -> None:
+    if status != SEED_OK:
+        msg = _lib.seed_status_string(status).decode()
+        raise SeedError(f"libseed status {status}: {msg}")
+
+
+@dataclass(frozen=True)
+class SeedConfig:
+    hq: int
+    hkv: int
+    head_dim: int
+    kmax: int
+    page_size: int = 16
+    scale: float = 0.0
+
+    def c(self) -> _Cfg:
+        return _Cfg(self.hq, self.hkv, self.head_dim, self.page_size, self.kmax, self.scale)
+
+
+@dataclass
+class PagedKV:
+    """One layer's cache: k, v bf16 [num_pages, hkv, page_size, head_dim];
+    page_table int32 [batch, max_pages]."""
+    k: torch.Tensor
+    v: torch.Tensor
+    page_table: torch.Tensor
+
+    def c(self) -> _KV:
+        return _KV(self.k.data_ptr(), self.v.data_ptr(), self.page_table.data_ptr(),
+                   self.page_table.shape[1], self.k.shape[0])
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def _t(x: torch.Tensor, dtype, shape, name: str) -> int:
+    if not isinstance(x, torch.Tensor):
+        raise TypeError(f"{name}: expected a torch.Tensor")
+    if x.dtype != dtype:
+        raise TypeError(f"{name}: dtype {x.dtype}, expected {dtype}")
+    if not x.is_cuda:
+        raise ValueError(f"{name}: must be a CUDA tensor")
+    if not x.is_contiguous():
+        raise ValueError(f"{name}: must be contiguous")
+    if shape is not None and tuple(x.shape) != tuple(shape):
+        raise ValueError(f"{name}: shape {tuple(x.shape)}, expected {tuple(shape)}")
+    return x.data_ptr()
+
+
+def _kv_checked(cfg: SeedConfig, kv: PagedKV, batch: int) -> _KV:
+    shp = (kv.k.shape[0], cfg.hkv, cfg.page_size, cfg.head_dim)
+    _t(kv.k, torch.bfloat16, shp, "kv.k")
+    _t(kv.v, torch.bfloat16, shp, "kv.v")
+    _t(kv.page_table, torch.int32, (batch, kv.page_table.shape[1]), "kv.page_table")
+    return kv.c()
+
+
+def seed_workspace_bytes(cfg: SeedConfig, batch: int) -> int:
+    c = cfg.c()
+    n = _lib.seed_workspace_bytes(ctypes.byref(c), batch)
+    if n == 0:
+        raise SeedError("invalid configuration")
+    return int(n)
+
+
+def new_workspace(cfg: SeedConfig, batch: int, device=None) -> torch.Tensor:
+    """A zero-filled workspace (uint8) for seed_draft_attn / seed_verify_attn."""
+    return torch.zeros(seed_workspace_bytes(cfg, batch), dtype=torch.uint8, device=device or "cuda")
+
+
+def seed_draft_kv_append(cfg: SeedConfig, k_new, v_new, draft_lens, draft_k, draft_v, err,
+                         stream=None) -> None:
+    B = draft_lens.shape[0]
+    c = cfg.c()
+    _check(_lib.seed_draft_kv_append(
+        ctypes.byref(c), B,
+        _t(k_new, torch.bfloat16, (B, cfg.hkv, cfg.head_dim), "k_new"),
+        _t(v_new, torch.bfloat16, (B, cfg.hkv, cfg.head_dim), "v_new"),
+        _t(draft_lens, torch.int32, (B,), "draft_lens"),
+        _t(draft_k, torch.bfloat16, (B, cfg.hkv, cfg.kmax, cfg.head_dim), "draft_k"),
+        _t(draft_v, torch.bfloat16, (B, cfg.hkv, cfg.kmax, cfg.head_dim), "draft_v"),
+        _t(err, torch.int32, (1,), "err"), _stream(stream)))
+
+
+def seed_draft_attn(cfg: SeedConfig, q, ctx_kv: PagedKV, draft_k, draft_v, ctx_lens, draft_lens,
+                    out, lse, ws, err, stream=None) -> None:
+    B = q.shape[0]
+    c = cfg.c()
+    _check(_lib.seed_draft_attn(
+        ctypes.byref(c), B,
+        _t(q, torch.bfloat16, (B, cfg.hq, cfg.head_dim), "q"),
+        _kv_checked(cfg, ctx_kv, B),
+        _t(draft_k, torch.bfloat16, (B, cfg.hkv, cfg.kmax, cfg.head_dim), "draft_k"),
+        _t(draft_v, torch.bfloat16, (B, cfg.hkv, cfg.kmax, cfg.head_dim), "draft_v"),
+        _t(ctx_lens, torch.int32, (B,), "ctx_lens"),
+        _t(draft_lens, torch.int32, (B,), "draft_lens"),
+        _t(out, torch.float32, (B, cfg.hq, cfg.head_dim), "out"),
+        _t(lse, torch.float32, (B, cfg.hq), "lse") if lse is not None else None,
+        _t(ws, torch.uint8, None, "ws"), ws.numel(),
+        _t(err, torch.int32, (1,), "err"), _stream(stream)))
+
+
+def seed_kv_append(cfg: SeedConfig, kv: PagedKV, k_new, v_new, n_new, ctx_lens, err,
+                   stream=None) -> None:
+    B = n_new.shape[0]
+    c = cfg.c()
+    shp = (B, cfg.kmax + 1, cfg.hkv, cfg.head_dim)
+    _check(_lib.seed_kv_append(
+        ctypes.byref(c), B, _kv_checked(cfg, kv, B),
+        _t(k_new, torch.bfloat16, shp, "k_new"), _t(v_new, torch.bfloat16, shp, "v_new"),
+        _t(n_new, torch.int32, (B,), "n_new"), _t(ctx_lens, torch.int32, (B,), "ctx_lens"),
+        _t(err, torch.int32, (1,), "err"), _stream(stream)))
+
+
+def seed_verify_attn(cfg: SeedConfig, q, n_q, kv: PagedKV, ctx_lens, out, lse, ws, err,
+                     stream=None) -> None:
+    B = q.shape[0]
+    c = cfg.c()
+    W = cfg.kmax + 1
+    _check(_lib.seed_verify_attn(
+        ctypes.byref(c), B,
+        _t(q, torch.bfloat16, (B, W, cfg.hq, cfg.head_dim), "q"),
+        _t(n_q, torch.int32, (B,), "n_q"),
+        _kv_checked(cfg, kv, B),
+        _t(ctx_lens, torch.int32, (B,), "ctx_lens"),
+        _t(out, torch.float32, (B, W, cfg.hq, cfg.head_dim), "out"),
+        _t(lse, torch.float32, (B, W, cfg.hq), "lse") if lse is not None else None,
+        _t(ws, torch.uint8, None, "ws"), ws.numel(),
+        _t(err, torch.int32, (1,), "err"), _stream(stream)))
+
+
+def seed_accept_commit(kmax: int, draft_ids, target_ids, k_b, page_table, page_size: int,
+                       ctx_lens, accepted, tokens, committed_slots, err, stream=None) -> None:
+    B = k_b.shape[0]
+    _check(_lib.seed_accept_commit(
+        B, kmax,
+        _t(draft_ids, torch.int32, (B, kmax), "draft_ids"),
+        _t(target_ids, torch.int32, (B, kmax + 1), "target_ids"),
+        _t(k_b, torch.int32, (B,), "k_b"),
+        _t(page_table, torch.int32, (B, page_table.shape[1]), "page_table"),
+        page_table.shape[1], page_size,
+        _t(ctx_lens, torch.int32, (B,), "ctx_lens"),
+        _t(accepted, torch.int32, (B,), "accepted"),
+        _t(tokens, torch.int32, (B, kmax + 1), "tokens"),
+        _t(committed_slots, torch.int32, (B, kmax + 1), "committed_slots"),
+        _t(err, torch.int32, (1,), "err"), _stream(stream)))
+
+
+def library() -> ctypes.CDLL:
+    """The loaded libseed.so (for ABI-level tests)."""
+    if _Lazy._cdll is None:
+        _Lazy._cdll = _load()
+    return _Lazy._cdll

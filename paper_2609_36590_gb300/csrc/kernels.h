@@ -1,0 +1,72 @@
+// Internal launch interface between the C ABI (seed_api.cu) and the kernels.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <cstddef>
+#include <cstdint>
+
+namespace seedk {
+
+constexpr int kPageTokens = 16;   // tokens per KV page; the only page size built
+
+// Split-KV flash-decoding work description (see decode_attn.cu).
+struct DecodeParams {
+  const uint16_t* q;          // bf16 [NV, hq, D]
+  const uint16_t* k_cache;    // bf16 [num_pages, hkv, 16, D]
+  const uint16_t* v_cache;
+  const int32_t* page_table;  // [B, max_pages]
+  int32_t max_pages;
+  int32_t num_pages;
+  const uint16_t* draft_k;    // bf16 [B, hkv, kmax, D] (draft mode only)
+  const uint16_t* draft_v;
+  const int32_t* ctx_lens;    // [B]
+  const int32_t* aux;         // draft: draft_lens [B]; verify: n_q [B]
+  float* out;                 // f32 [NV, hq, D]
+  float* lse;                 // f32 [NV, hq] or null
+  float* part;                // split partial records
+  int32_t* counters;          // [NV * hkv] arrival counters (zero between calls)
+  int32_t* err;
+  int32_t B, hq, hkv, kmax;
+  int32_t nq_per_seq;         // virtual sequences per real sequence: 1 or kmax+1
+  int32_t verify;             // 0: draft rows after the context; 1: causal verify
+  int32_t ppu;                // pages per work unit (multiple of 4)
+  int32_t cmax;               // work units per (virtual sequence, KV head)
+  int32_t n_units;            // NV * hkv * cmax
+  float scale_log2;           // softmax scale * log2(e)
+};
+
+// Work split shared by the host-side planner and the workspace-size bound.
+constexpr int kTargetUnits = 2048;
+
+struct DecodePlan {
+  int32_t nv, ppu, cmax, n_units;
+  size_t counters_bytes, part_bytes;
+};
+
+DecodePlan plan_decode(int32_t nv, int32_t hkv, int32_t group, int32_t head_dim,
+                       int32_t max_pages);
+size_t decode_workspace_bound(int32_t nv_max, int32_t hkv, int32_t group, int32_t head_dim);
+
+cudaError_t launch_decode(const DecodeParams& p, int head_dim, int group, cudaStream_t st);
+
+cudaError_t launch_draft_append(int32_t B, int32_t hkv, int32_t head_dim, int32_t kmax,
+                                const uint16_t* k_new, const uint16_t* v_new,
+                                const int32_t* draft_lens, uint16_t* draft_k, uint16_t* draft_v,
+                                int32_t* err, cudaStream_t st);
+
+cudaError_t launch_kv_append(int32_t B, int32_t hkv, int32_t head_dim, int32_t kmax,
+                             uint16_t* k_cache, uint16_t* v_cache, const int32_t* page_table,
+                             int32_t max_pages, int32_t num_pages, const uint16_t* k_new,
+                             const uint16_t* v_new, const int32_t* n_new,
+                             const int32_t* ctx_lens, int32_t* err, cudaStream_t st);
+
+cudaError_t launch_accept(int32_t B, int32_t kmax, const int32_t* draft_ids,
+                          const int32_t* target_ids, const int32_t* k_b,
+                          const int32_t* page_table, int32_t max_pages, int32_t page_size,
+                          int32_t* ctx_lens, int32_t* accepted, int32_t* tokens,
+                          int32_t* slots, int32_t* err, cudaStream_t st);
+
+int device_sm_count();
+
+}  // namespace seedk

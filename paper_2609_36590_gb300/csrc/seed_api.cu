@@ -1,0 +1,206 @@
+// The C ABI of include/seed.h: host-side argument checks, work planning and
+// kernel launches.  No allocation, no synchronisation, no state.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdint>
+
+#include "../../include/seed.h"
+#include "kernels.h"
+
+namespace {
+
+constexpr size_t kAlign = 256;
+
+size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+bool group_supported(int g) { return g == 1 || g == 2 || g == 4 || g == 8; }
+
+seed_status_t check_cfg(const seed_cfg_t* cfg) {
+  if (cfg == nullptr) return SEED_ERR_NULL;
+  if (cfg->hq <= 0 || cfg->hkv <= 0 || cfg->hq % cfg->hkv != 0) return SEED_ERR_SHAPE;
+  if (cfg->kmax < 1 || cfg->kmax > SEED_MAX_KMAX) return SEED_ERR_SHAPE;
+  if (!(cfg->scale >= 0.f) || std::isinf(cfg->scale)) return SEED_ERR_SHAPE;
+  if (cfg->head_dim != 64 && cfg->head_dim != 128) return SEED_ERR_UNSUPPORTED;
+  if (!group_supported(cfg->hq / cfg->hkv)) return SEED_ERR_UNSUPPORTED;
+  if (cfg->page_size != seedk::kPageTokens) return SEED_ERR_UNSUPPORTED;
+  return SEED_OK;
+}
+
+seed_status_t check_kv(const seed_kv_t& kv) {
+  if (kv.k == nullptr || kv.v == nullptr || kv.page_table == nullptr) return SEED_ERR_NULL;
+  if (kv.max_pages <= 0 || kv.num_pages <= 0) return SEED_ERR_RANGE;
+  if ((long long)kv.max_pages * seedk::kPageTokens > INT32_MAX) return SEED_ERR_RANGE;
+  return SEED_OK;
+}
+
+float scale_of(const seed_cfg_t* cfg) {
+  return cfg->scale > 0.f ? cfg->scale : 1.0f / std::sqrt((float)cfg->head_dim);
+}
+
+// Workspace layout: arrival counters for batch*(kmax+1)*hkv (virtual
+// sequence, KV head) pairs, then the split partial records.
+size_t counters_bytes(const seed_cfg_t* cfg, int32_t batch) {
+  return round_up((size_t)batch * (cfg->kmax + 1) * cfg->hkv * sizeof(int32_t), kAlign);
+}
+
+seed_status_t finish(cudaError_t e) { return e == cudaSuccess ? SEED_OK : SEED_ERR_CUDA; }
+
+seed_status_t run_decode(const seed_cfg_t* cfg, int32_t batch, bool verify, const void* q,
+                         const seed_kv_t& kv, const void* draft_k, const void* draft_v,
+                         const int32_t* ctx_lens, const int32_t* aux, float* out, float* lse,
+                         void* ws, size_t ws_bytes, int32_t* err, void* stream) {
+  const int G = cfg->hq / cfg->hkv;
+  const int nq = verify ? cfg->kmax + 1 : 1;
+  const int nv = batch * nq;
+  const seedk::DecodePlan pl = seedk::plan_decode(nv, cfg->hkv, G, cfg->head_dim, kv.max_pages);
+  const size_t cb = counters_bytes(cfg, batch);
+  if (ws_bytes < cb + pl.part_bytes) return SEED_ERR_WORKSPACE;
+  seedk::DecodeParams p{};
+  p.q = static_cast<const uint16_t*>(q);
+  p.k_cache = static_cast<const uint16_t*>(kv.k);
+  p.v_cache = static_cast<const uint16_t*>(kv.v);
+  p.page_table = kv.page_table;
+  p.max_pages = kv.max_pages;
+  p.num_pages = kv.num_pages;
+  p.draft_k = static_cast<const uint16_t*>(draft_k);
+  p.draft_v = static_cast<const uint16_t*>(draft_v);
+  p.ctx_lens = ctx_lens;
+  p.aux = aux;
+  p.out = out;
+  p.lse = lse;
+  p.counters = static_cast<int32_t*>(ws);
+  p.part = reinterpret_cast<float*>(static_cast<char*>(ws) + cb);
+  p.err = err;
+  p.B = batch;
+  p.hq = cfg->hq;
+  p.hkv = cfg->hkv;
+  p.kmax = cfg->kmax;
+  p.nq_per_seq = nq;
+  p.verify = verify ? 1 : 0;
+  p.ppu = pl.ppu;
+  p.cmax = pl.cmax;
+  p.n_units = pl.n_units;
+  p.scale_log2 = scale_of(cfg) * 1.4426950408889634f;
+  return finish(seedk::launch_decode(p, cfg->head_dim, G, static_cast<cudaStream_t>(stream)));
+}
+
+bool misaligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) != 0; }
+
+}  // namespace
+
+extern "C" {
+
+int32_t seed_abi_version(void) { return SEED_ABI_VERSION; }
+
+const char* seed_status_string(seed_status_t s) {
+  switch (s) {
+    case SEED_OK: return "ok";
+    case SEED_ERR_NULL: return "a required pointer is NULL";
+    case SEED_ERR_SHAPE: return "invalid shape (batch, heads or kmax)";
+    case SEED_ERR_RANGE: return "max_pages / num_pages out of range";
+    case SEED_ERR_UNSUPPORTED: return "head_dim, group size or page_size not supported";
+    case SEED_ERR_CUDA: return "CUDA launch failed";
+    case SEED_ERR_WORKSPACE: return "workspace too small or misaligned";
+  }
+  return "unknown status";
+}
+
+size_t seed_workspace_bytes(const seed_cfg_t* cfg, int32_t batch) {
+  if (check_cfg(cfg) != SEED_OK || batch < 0) return 0;
+  const int G = cfg->hq / cfg->hkv;
+  const int32_t nv_max = batch * (cfg->kmax + 1);
+  return counters_bytes(cfg, batch) +
+         round_up(seedk::decode_workspace_bound(nv_max, cfg->hkv, G, cfg->head_dim), kAlign);
+}
+
+seed_status_t seed_draft_kv_append(const seed_cfg_t* cfg, int32_t batch, const void* k_new,
+                                   const void* v_new, const int32_t* draft_lens, void* draft_k,
+                                   void* draft_v, int32_t* err_flag, void* stream) {
+  seed_status_t st = check_cfg(cfg);
+  if (st != SEED_OK) return st;
+  if (batch < 0) return SEED_ERR_SHAPE;
+  if (batch == 0) return SEED_OK;
+  if (!k_new || !v_new || !draft_lens || !draft_k || !draft_v || !err_flag) return SEED_ERR_NULL;
+  if (misaligned16(k_new) || misaligned16(v_new) || misaligned16(draft_k) || misaligned16(draft_v))
+    return SEED_ERR_RANGE;
+  return finish(seedk::launch_draft_append(
+      batch, cfg->hkv, cfg->head_dim, cfg->kmax, static_cast<const uint16_t*>(k_new),
+      static_cast<const uint16_t*>(v_new), draft_lens, static_cast<uint16_t*>(draft_k),
+      static_cast<uint16_t*>(draft_v), err_flag, static_cast<cudaStream_t>(stream)));
+}
+
+seed_status_t seed_draft_attn(const seed_cfg_t* cfg, int32_t batch, const void* q,
+                              seed_kv_t ctx_kv, const void* draft_k, const void* draft_v,
+                              const int32_t* ctx_lens, const int32_t* draft_lens, float* out,
+                              float* lse, void* ws, size_t ws_bytes, int32_t* err_flag,
+                              void* stream) {
+  seed_status_t st = check_cfg(cfg);
+  if (st != SEED_OK) return st;
+  if (batch < 0) return SEED_ERR_SHAPE;
+  if (batch == 0) return SEED_OK;
+  if (!q || !draft_k || !draft_v || !ctx_lens || !draft_lens || !out || !ws || !err_flag)
+    return SEED_ERR_NULL;
+  if ((st = check_kv(ctx_kv)) != SEED_OK) return st;
+  if (misaligned16(q) || misaligned16(ctx_kv.k) || misaligned16(ctx_kv.v) ||
+      misaligned16(draft_k) || misaligned16(draft_v))
+    return SEED_ERR_RANGE;
+  if ((reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)) != 0) return SEED_ERR_WORKSPACE;
+  return run_decode(cfg, batch, false, q, ctx_kv, draft_k, draft_v, ctx_lens, draft_lens, out, lse,
+                    ws, ws_bytes, err_flag, stream);
+}
+
+seed_status_t seed_kv_append(const seed_cfg_t* cfg, int32_t batch, seed_kv_t kv,
+                             const void* k_new, const void* v_new, const int32_t* n_new,
+                             const int32_t* ctx_lens, int32_t* err_flag, void* stream) {
+  seed_status_t st = check_cfg(cfg);
+  if (st != SEED_OK) return st;
+  if (batch < 0) return SEED_ERR_SHAPE;
+  if (batch == 0) return SEED_OK;
+  if (!k_new || !v_new || !n_new || !ctx_lens || !err_flag) return SEED_ERR_NULL;
+  if ((st = check_kv(kv)) != SEED_OK) return st;
+  if (misaligned16(k_new) || misaligned16(v_new) || misaligned16(kv.k) || misaligned16(kv.v))
+    return SEED_ERR_RANGE;
+  return finish(seedk::launch_kv_append(
+      batch, cfg->hkv, cfg->head_dim, cfg->kmax, static_cast<uint16_t*>(kv.k),
+      static_cast<uint16_t*>(kv.v), kv.page_table, kv.max_pages, kv.num_pages,
+      static_cast<const uint16_t*>(k_new), static_cast<const uint16_t*>(v_new), n_new, ctx_lens,
+      err_flag, static_cast<cudaStream_t>(stream)));
+}
+
+seed_status_t seed_verify_attn(const seed_cfg_t* cfg, int32_t batch, const void* q,
+                               const int32_t* n_q, seed_kv_t kv, const int32_t* ctx_lens,
+                               float* out, float* lse, void* ws, size_t ws_bytes,
+                               int32_t* err_flag, void* stream) {
+  seed_status_t st = check_cfg(cfg);
+  if (st != SEED_OK) return st;
+  if (batch < 0) return SEED_ERR_SHAPE;
+  if (batch == 0) return SEED_OK;
+  if (!q || !n_q || !ctx_lens || !out || !ws || !err_flag) return SEED_ERR_NULL;
+  if ((st = check_kv(kv)) != SEED_OK) return st;
+  if (misaligned16(q) || misaligned16(kv.k) || misaligned16(kv.v)) return SEED_ERR_RANGE;
+  if ((reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)) != 0) return SEED_ERR_WORKSPACE;
+  return run_decode(cfg, batch, true, q, kv, nullptr, nullptr, ctx_lens, n_q, out, lse, ws,
+                    ws_bytes, err_flag, stream);
+}
+
+seed_status_t seed_accept_commit(int32_t batch, int32_t kmax, const int32_t* draft_ids,
+                                 const int32_t* target_ids, const int32_t* k_b,
+                                 const int32_t* page_table, int32_t max_pages,
+                                 int32_t page_size, int32_t* ctx_lens, int32_t* accepted,
+                                 int32_t* tokens, int32_t* committed_slots, int32_t* err_flag,
+                                 void* stream) {
+  if (batch < 0 || kmax < 1 || kmax > SEED_MAX_KMAX) return SEED_ERR_SHAPE;
+  if (batch == 0) return SEED_OK;
+  if (!draft_ids || !target_ids || !k_b || !page_table || !ctx_lens || !accepted || !tokens ||
+      !committed_slots || !err_flag)
+    return SEED_ERR_NULL;
+  if (max_pages <= 0 || page_size <= 0 || (long long)max_pages * page_size > INT32_MAX)
+    return SEED_ERR_RANGE;
+  return finish(seedk::launch_accept(batch, kmax, draft_ids, target_ids, k_b, page_table,
+                                     max_pages, page_size, ctx_lens, accepted, tokens,
+                                     committed_slots, err_flag,
+                                     static_cast<cudaStream_t>(stream)));
+}
+
+}  // extern "C"

@@ -1,0 +1,134 @@
+"""The C ABI without a GPU: libseed.so loads, exports every function that
+include/seed.h declares, and its host-side checks return the documented
+statuses before touching CUDA (null pointers, unsupported shapes, bad page
+ranges, small or misaligned workspaces, empty batches)."""
+
+import ctypes
+import os
+import re
+import subprocess
+
+import pytest
+
+import paper_2609_36590_gb300 as seed
+from paper_2609_36590_gb300 import _Cfg, _KV, build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "seed.h")
+
+OK, ERR_NULL, ERR_SHAPE, ERR_RANGE, ERR_UNSUP, ERR_CUDA, ERR_WS = range(7)
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return seed.library()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(seed_[a-z_]+)\s*\(", text)))
+
+
+def test_exports_every_declared_function(lib):
+    names = declared_functions()
+    assert len(names) >= 8
+    out = subprocess.run(["nm", "-D", "--defined-only", seed.LIB_PATH], capture_output=True,
+                         text=True, check=True).stdout
+    exported = set(re.findall(r"\bT (seed_\w+)", out))
+    missing = [n for n in names if n not in exported]
+    assert not missing, missing
+    for n in names:
+        assert hasattr(lib, n)
+
+
+def test_version_and_strings(lib):
+    assert lib.seed_abi_version() == 1
+    for s in range(7):
+        assert len(lib.seed_status_string(s)) > 0
+    assert lib.seed_status_string(99) == b"unknown status"
+
+
+def cfg(**kw):
+    base = dict(hq=32, hkv=8, head_dim=128, page_size=16, kmax=4, scale=0.0)
+    base.update(kw)
+    return _Cfg(**base)
+
+
+@pytest.mark.parametrize("kw,expect", [
+    (dict(), OK), (dict(head_dim=96), ERR_UNSUP), (dict(hq=24, hkv=8), ERR_UNSUP),
+    (dict(hq=30, hkv=8), ERR_SHAPE), (dict(kmax=0), ERR_SHAPE), (dict(kmax=17), ERR_SHAPE),
+    (dict(page_size=32), ERR_UNSUP), (dict(scale=-1.0), ERR_SHAPE), (dict(head_dim=64), OK),
+])
+def test_workspace_bytes_validates_cfg(lib, kw, expect):
+    c = cfg(**kw)
+    n = lib.seed_workspace_bytes(ctypes.byref(c), 4)
+    assert (n > 0) == (expect == OK)
+
+
+def test_workspace_grows_with_batch(lib):
+    c = cfg()
+    sizes = [lib.seed_workspace_bytes(ctypes.byref(c), b) for b in (1, 16, 64)]
+    assert sizes[0] < sizes[1] < sizes[2]
+    assert all(s % 256 == 0 for s in sizes)
+
+
+FAKE = 0x10000  # never dereferenced: every call below fails a host check first
+
+
+def kv(**kw):
+    base = dict(k=FAKE, v=FAKE, page_table=FAKE, max_pages=8, num_pages=8)
+    base.update(kw)
+    return _KV(**base)
+
+
+def draft_call(lib, c, B=1, q=FAKE, k=None, ws=FAKE, ws_bytes=1 << 30, err=FAKE, out=FAKE):
+    return lib.seed_draft_attn(ctypes.byref(c), B, q, k or kv(), FAKE, FAKE, FAKE, FAKE, out,
+                               None, ws, ws_bytes, err, None)
+
+
+def test_draft_attn_host_checks(lib):
+    c = cfg()
+    assert draft_call(lib, c, B=0) == OK                 # empty batch: nothing launched
+    assert draft_call(lib, c, B=-1) == ERR_SHAPE
+    assert draft_call(lib, c, q=None) == ERR_NULL
+    assert draft_call(lib, c, out=None) == ERR_NULL
+    assert draft_call(lib, c, err=None) == ERR_NULL
+    assert draft_call(lib, c, k=kv(k=None)) == ERR_NULL
+    assert draft_call(lib, c, k=kv(max_pages=0)) == ERR_RANGE
+    assert draft_call(lib, c, k=kv(num_pages=0)) == ERR_RANGE
+    assert draft_call(lib, c, q=FAKE + 8) == ERR_RANGE   # not 16-byte aligned
+    assert draft_call(lib, c, ws=FAKE + 128) == ERR_WS   # not 256-byte aligned
+    assert draft_call(lib, c, ws_bytes=16) == ERR_WS
+    bad = cfg(head_dim=80)
+    assert draft_call(lib, bad) == ERR_UNSUP
+
+
+def test_verify_and_append_host_checks(lib):
+    c = cfg()
+    assert lib.seed_verify_attn(ctypes.byref(c), 0, FAKE, FAKE, kv(), FAKE, FAKE, None, FAKE,
+                                1 << 30, FAKE, None) == OK
+    assert lib.seed_verify_attn(ctypes.byref(c), 2, FAKE, None, kv(), FAKE, FAKE, None, FAKE,
+                                1 << 30, FAKE, None) == ERR_NULL
+    assert lib.seed_verify_attn(ctypes.byref(c), 2, FAKE, FAKE, kv(), FAKE, FAKE, None, FAKE,
+                                64, FAKE, None) == ERR_WS
+    assert lib.seed_kv_append(ctypes.byref(c), 2, kv(), FAKE, FAKE, None, FAKE, FAKE,
+                              None) == ERR_NULL
+    assert lib.seed_kv_append(ctypes.byref(c), 2, kv(max_pages=-3), FAKE, FAKE, FAKE, FAKE, FAKE,
+                              None) == ERR_RANGE
+    assert lib.seed_draft_kv_append(ctypes.byref(c), 2, FAKE, None, FAKE, FAKE, FAKE, FAKE,
+                                    None) == ERR_NULL
+    assert lib.seed_draft_kv_append(ctypes.byref(c), 0, None, None, None, None, None, None,
+                                    None) == OK
+
+
+def test_accept_host_checks(lib):
+    args = [FAKE] * 4 + [8, 16] + [FAKE] * 5
+    assert lib.seed_accept_commit(0, 4, *args, None) == OK
+    assert lib.seed_accept_commit(2, 0, *args, None) == ERR_SHAPE
+    assert lib.seed_accept_commit(2, 17, *args, None) == ERR_SHAPE
+    bad = [FAKE, None] + args[2:]
+    assert lib.seed_accept_commit(2, 4, *bad, None) == ERR_NULL
+    bad = args[:4] + [0, 16] + args[6:]
+    assert lib.seed_accept_commit(2, 4, *bad, None) == ERR_RANGE

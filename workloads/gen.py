@@ -209,3 +209,65 @@ def round_plan(wl: Workload, rnd: int):
         draft[b, kb:] = target[b, kb:K]
     return (k_b.astype(np.int32), n.astype(np.int32),
             draft.astype(np.int32), target.astype(np.int32))
+
+
+# ---------------------------------------------------------------- small cases
+def small_case(seed: int, B: int, hq: int, hkv: int, D: int, kmax: int, max_ctx: int,
+               paged_random: bool = True, key_scale: float = 1.0) -> dict:
+    """A random problem small enough for the oracle to check every output.
+
+    Lengths cover the edges (0, 1, a page minus/plus one, multiples of the
+    page) when B is large enough.  Returns uint16 bf16 bits for all tensors:
+      rows_k/rows_v [B, max_ctx+kmax+1, hkv, D]  logical cache rows by position
+      q_draft [B, hq, D], q_verify [B, kmax+1, hq, D]
+      draft_k/draft_v [B, hkv, kmax, D]
+    and int32 lens [B], draft_lens [B] (0..kmax), n_q [B] (0..kmax+1),
+    page_table [B, max_pages], max_pages.
+    """
+    g = rng(9000, seed)
+    edges = [0, 1, PAGE_SIZE - 1, PAGE_SIZE, PAGE_SIZE + 1, 2 * PAGE_SIZE, max_ctx]
+    lens = g.integers(0, max_ctx + 1, size=B)
+    for i in range(min(B, len(edges))):
+        lens[i] = min(edges[i], max_ctx)
+    n_q = g.integers(1, kmax + 2, size=B)
+    draft_lens = g.integers(1, kmax + 1, size=B)
+    if B >= 3:
+        n_q[B - 1] = 0                      # a sequence that skips the verify call
+        draft_lens[B - 2] = 0               # ... and one that skips the draft call
+    n_rows = max_ctx + kmax + 1
+    max_pages = -(-n_rows // PAGE_SIZE) + 1
+    perm = g.permutation(B * max_pages) if paged_random else np.arange(B * max_pages)
+    pt = perm.reshape(B, max_pages)
+
+    def bits(shape, s=1.0):
+        return f32_to_bf16_bits(g.standard_normal(shape, dtype=np.float32) * np.float32(s))
+
+    return dict(
+        lens=lens.astype(np.int32), n_q=n_q.astype(np.int32),
+        draft_lens=draft_lens.astype(np.int32), page_table=pt.astype(np.int32),
+        max_pages=max_pages,
+        rows_k=bits((B, n_rows, hkv, D), key_scale), rows_v=bits((B, n_rows, hkv, D)),
+        q_draft=bits((B, hq, D)), q_verify=bits((B, kmax + 1, hq, D)),
+        draft_k=bits((B, hkv, kmax, D)), draft_v=bits((B, hkv, kmax, D)))
+
+
+def accept_case(seed: int, B: int, kmax: int, vocab: int = 50, max_ctx: int = 300) -> dict:
+    """Random acceptance inputs: k_b in 0..kmax, token ids with a planned first
+    mismatch (sometimes none), positions past k_b equal to the target (so a
+    reader that ignores k_b over-accepts), lengths and a page permutation."""
+    g = rng(9100, seed)
+    k_b = g.integers(0, kmax + 1, size=B)
+    target = g.integers(0, vocab, size=(B, kmax + 1))
+    draft = g.integers(0, vocab, size=(B, kmax))
+    for b in range(B):
+        n = int(g.integers(0, k_b[b] + 1))
+        draft[b, :n] = target[b, :n]
+        if n < k_b[b]:
+            draft[b, n] = (target[b, n] + 1 + g.integers(0, vocab - 1)) % vocab
+        draft[b, k_b[b]:] = target[b, k_b[b]:kmax]
+    lens = g.integers(0, max_ctx + 1, size=B)
+    max_pages = -(-(max_ctx + kmax + 1) // PAGE_SIZE)
+    pt = g.permutation(B * max_pages).reshape(B, max_pages)
+    return dict(k_b=k_b.astype(np.int32), draft_ids=draft.astype(np.int32),
+                target_ids=target.astype(np.int32), lens=lens.astype(np.int32),
+                page_table=pt.astype(np.int32), max_pages=max_pages)
