@@ -292,7 +292,7 @@ def run_e2e(dw, wl, stream, W, K, lens):
         vq=torch.empty(len(dw.layers), B, Km + 1, Hq, D, dtype=torch.bfloat16, device=dev),
         vk=torch.empty(len(dw.layers), B, Km + 1, Hkv, D, dtype=torch.bfloat16, device=dev),
         vv=torch.empty(len(dw.layers), B, Km + 1, Hkv, D, dtype=torch.bfloat16, device=dev),
-        ints=torch.empty(steps + 2 + Km + (Km + 1), B, dtype=torch.int32, device=dev))
+        ints=torch.empty(steps + 2, B, dtype=torch.int32, device=dev))
     ints = st["ints"]
     ins = dict(steps=steps, draft_lens=[ints[i] for i in range(steps)], k_b=ints[steps],
                n_q=ints[steps + 1])

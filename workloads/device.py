@@ -23,7 +23,7 @@ from .configs import PAGE_SIZE, Workload
 
 
 def bf16_tensor(bits: np.ndarray, device) -> torch.Tensor:
-    return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).to(device).view(torch.bfloat16)
+    return torch.from_numpy(np.array(bits, copy=True).view(np.int16)).to(device).view(torch.bfloat16)
 
 
 class DeviceWorkload:
