@@ -69,4 +69,30 @@ cudaError_t launch_accept(int32_t B, int32_t kmax, const int32_t* draft_ids,
 
 int device_sm_count();
 
+// Tensor-core verify attention (verify_tc.cu).
+constexpr int kTcUnitsCap = 1024;   // most work units one verify launch plans
+
+struct VerifyTcParams {
+  const int32_t* page_table;
+  int32_t max_pages;
+  int32_t num_pages;
+  const int32_t* ctx_lens;    // [B]
+  const int32_t* n_q;         // [B]
+  float* out;                 // f32 [B, kmax+1, hq, 128]
+  float* lse;                 // f32 [B, kmax+1, hq] or null
+  float* part;                // partial records
+  int32_t* counters;          // [B * hkv] arrival counters (zero between calls)
+  int32_t* sched;             // [2] unit dispenser and finished-CTA count (zero between calls)
+  int32_t* err;
+  int32_t B, hq, hkv, kmax, G;
+  int32_t target_units;
+  float scale_log2;
+};
+
+bool verify_tc_supported(int head_dim, int group, int kmax);
+int verify_tc_target_units();
+size_t verify_tc_part_bound(int32_t batch, int32_t hkv, int32_t group, int32_t kmax);
+cudaError_t launch_verify_tc(const VerifyTcParams& p, const void* q, const void* k_cache,
+                             const void* v_cache, cudaStream_t st);
+
 }  // namespace seedk

@@ -2,6 +2,7 @@
 // kernel launches.  No allocation, no synchronisation, no state.
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdint>
 
@@ -38,8 +39,11 @@ float scale_of(const seed_cfg_t* cfg) {
   return cfg->scale > 0.f ? cfg->scale : 1.0f / std::sqrt((float)cfg->head_dim);
 }
 
-// Workspace layout: arrival counters for batch*(kmax+1)*hkv (virtual
-// sequence, KV head) pairs, then the split partial records.
+// Workspace layout: [0, 256) the tensor-core verify's unit dispenser; then
+// arrival counters for batch*(kmax+1)*hkv (virtual sequence, KV head) pairs;
+// then the split partial records.  Every kernel leaves the counters at zero.
+constexpr size_t kSchedBytes = kAlign;
+
 size_t counters_bytes(const seed_cfg_t* cfg, int32_t batch) {
   return round_up((size_t)batch * (cfg->kmax + 1) * cfg->hkv * sizeof(int32_t), kAlign);
 }
@@ -54,7 +58,7 @@ seed_status_t run_decode(const seed_cfg_t* cfg, int32_t batch, bool verify, cons
   const int nq = verify ? cfg->kmax + 1 : 1;
   const int nv = batch * nq;
   const seedk::DecodePlan pl = seedk::plan_decode(nv, cfg->hkv, G, cfg->head_dim, kv.max_pages);
-  const size_t cb = counters_bytes(cfg, batch);
+  const size_t cb = kSchedBytes + counters_bytes(cfg, batch);
   if (ws_bytes < cb + pl.part_bytes) return SEED_ERR_WORKSPACE;
   seedk::DecodeParams p{};
   p.q = static_cast<const uint16_t*>(q);
@@ -69,7 +73,7 @@ seed_status_t run_decode(const seed_cfg_t* cfg, int32_t batch, bool verify, cons
   p.aux = aux;
   p.out = out;
   p.lse = lse;
-  p.counters = static_cast<int32_t*>(ws);
+  p.counters = reinterpret_cast<int32_t*>(static_cast<char*>(ws) + kSchedBytes);
   p.part = reinterpret_cast<float*>(static_cast<char*>(ws) + cb);
   p.err = err;
   p.B = batch;
@@ -83,6 +87,40 @@ seed_status_t run_decode(const seed_cfg_t* cfg, int32_t batch, bool verify, cons
   p.n_units = pl.n_units;
   p.scale_log2 = scale_of(cfg) * 1.4426950408889634f;
   return finish(seedk::launch_decode(p, cfg->head_dim, G, static_cast<cudaStream_t>(stream)));
+}
+
+// Verify attention on the tensor cores (head_dim 128, all G*(kmax+1) query
+// rows of a KV head in one 128-row tile).
+seed_status_t run_verify_tc(const seed_cfg_t* cfg, int32_t batch, const void* q,
+                            const int32_t* n_q, const seed_kv_t& kv, const int32_t* ctx_lens,
+                            float* out, float* lse, void* ws, size_t ws_bytes, int32_t* err,
+                            void* stream) {
+  const int G = cfg->hq / cfg->hkv;
+  const size_t cb = kSchedBytes + counters_bytes(cfg, batch);
+  const int target = seedk::verify_tc_target_units();
+  const size_t need = cb + ((size_t)target + (size_t)batch * cfg->hkv) * G * (cfg->kmax + 1) *
+                               (cfg->head_dim + 1) * sizeof(float);
+  if (ws_bytes < need) return SEED_ERR_WORKSPACE;
+  seedk::VerifyTcParams p{};
+  p.page_table = kv.page_table;
+  p.max_pages = kv.max_pages;
+  p.num_pages = kv.num_pages;
+  p.ctx_lens = ctx_lens;
+  p.n_q = n_q;
+  p.out = out;
+  p.lse = lse;
+  p.sched = static_cast<int32_t*>(ws);
+  p.counters = reinterpret_cast<int32_t*>(static_cast<char*>(ws) + kSchedBytes);
+  p.part = reinterpret_cast<float*>(static_cast<char*>(ws) + cb);
+  p.err = err;
+  p.B = batch;
+  p.hq = cfg->hq;
+  p.hkv = cfg->hkv;
+  p.kmax = cfg->kmax;
+  p.G = G;
+  p.target_units = target;
+  p.scale_log2 = scale_of(cfg) * 1.4426950408889634f;
+  return finish(seedk::launch_verify_tc(p, q, kv.k, kv.v, static_cast<cudaStream_t>(stream)));
 }
 
 bool misaligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) != 0; }
@@ -110,8 +148,10 @@ size_t seed_workspace_bytes(const seed_cfg_t* cfg, int32_t batch) {
   if (check_cfg(cfg) != SEED_OK || batch < 0) return 0;
   const int G = cfg->hq / cfg->hkv;
   const int32_t nv_max = batch * (cfg->kmax + 1);
-  return counters_bytes(cfg, batch) +
-         round_up(seedk::decode_workspace_bound(nv_max, cfg->hkv, G, cfg->head_dim), kAlign);
+  size_t part = seedk::decode_workspace_bound(nv_max, cfg->hkv, G, cfg->head_dim);
+  if (seedk::verify_tc_supported(cfg->head_dim, G, cfg->kmax))
+    part = std::max(part, seedk::verify_tc_part_bound(batch, cfg->hkv, G, cfg->kmax));
+  return kSchedBytes + counters_bytes(cfg, batch) + round_up(part, kAlign);
 }
 
 seed_status_t seed_draft_kv_append(const seed_cfg_t* cfg, int32_t batch, const void* k_new,
@@ -180,6 +220,9 @@ seed_status_t seed_verify_attn(const seed_cfg_t* cfg, int32_t batch, const void*
   if ((st = check_kv(kv)) != SEED_OK) return st;
   if (misaligned16(q) || misaligned16(kv.k) || misaligned16(kv.v)) return SEED_ERR_RANGE;
   if ((reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)) != 0) return SEED_ERR_WORKSPACE;
+  if (seedk::verify_tc_supported(cfg->head_dim, cfg->hq / cfg->hkv, cfg->kmax))
+    return run_verify_tc(cfg, batch, q, n_q, kv, ctx_lens, out, lse, ws, ws_bytes, err_flag,
+                         stream);
   return run_decode(cfg, batch, true, q, kv, nullptr, nullptr, ctx_lens, n_q, out, lse, ws,
                     ws_bytes, err_flag, stream);
 }
