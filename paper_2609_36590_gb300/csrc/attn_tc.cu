@@ -1,0 +1,781 @@
+// Draft and verify attention on the 5th-generation tensor cores (tcgen05,
+// TMEM, TMA).
+//
+// What it computes (Sec. 4.1: the drafter's cross-attention is ordinary
+// self-attention over the cache; Alg. 2 fixes the visible rows), for sequence
+// b and each of the G query heads of KV head g:
+//   verify: query j < n_q[b] (token X_draft[j]) over cache rows 0 .. L + j,
+//           L = ctx_lens[b] (the cache already holds the n_q new rows);
+//   draft:  one query over cache rows 0 .. L - 1 (the deep KV the last
+//           verification left) followed by draft rows 0 .. nd - 1 of the
+//           draft scratch (X_draft[0 .. nd-1], the query's own row included).
+//
+// Design.  All G * n_q query rows of one (sequence, KV head) sit in the rows
+// of one M=128 MMA tile, so every K/V byte is read from HBM once per call
+// whatever k is.  A sequence is a list of 16-token pages (cache pages, then for
+// the draft one page holding the draft rows); 8 pages make a 128-token tile
+// that flows through a 3-stage TMA ring (128-byte swizzled boxes of one page x
+// 64 head dims).  Per tile one thread issues S = Q K^T (8 MMAs, M=128 N=128
+// K=16) into a double-buffered TMEM accumulator; four softmax warps (one per
+// TMEM lane quarter, one thread per query row) read S, mask it per column,
+// run the online softmax in log2 units (the output accumulator is rescaled
+// only when the running maximum grows by more than 2^8) and write the
+// probabilities back into the same TMEM columns as two bf16 halves
+// P = P_hi + P_lo (P_hi = bf16(P), P_lo = bf16(P - P_hi)); the MMA thread
+// then accumulates O += P_hi V + P_lo V with A read from TMEM and V read
+// MN-major from shared memory.  The two-term split keeps ~16 bits of each
+// probability, enough for 2e-3 absolute accuracy on the peaked rows of the
+// x8-key workload (one bf16 term alone is not).  V rows of columns that no
+// query may see (past the sequence end, unfilled page slots) are zeroed in
+// shared memory before PV so that stale or poisoned rows contribute nothing.
+//
+// Work: units of `tpu` tiles of one (b, g) are handed out by an atomic
+// counter, full-size units first and ragged ones last.  Units of the same
+// (b, g) leave normalised partials and log2-sum-exps (column-major, so stores
+// and loads coalesce across the rows); per TMEM lane quarter the last warp to
+// finish merges them in unit order, so results are deterministic.
+//
+// Warp roles (192 threads): warp 0 TMA producer and scheduler, warp 1 MMA
+// issuer and TMEM owner, warps 2-5 softmax / epilogue.  Every wait is bounded;
+// a wait that gives up raises SEED_DEVERR_TIMEOUT and all roles drain out.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <atomic>
+#include <cmath>
+#include <mutex>
+
+#include "common.cuh"
+#include "kernels.h"
+#include "tc.cuh"
+
+namespace seedk {
+namespace {
+
+constexpr int kD = 128;
+constexpr int kN = 128;                      // tokens (columns) per tile
+constexpr int kPagesPerTile = kN / kPage;    // 8
+constexpr int kStagesTC = 3;
+constexpr int kThreadsTC = 192;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kColO = 256;              // O accumulator columns [256, 384)
+constexpr float kRescale = 8.0f;
+constexpr float kLn2 = 0.69314718055994531f;
+constexpr unsigned kFull = 0xffffffffu;
+
+constexpr uint32_t kHalf = kN * 128;                   // 16 KiB: 128 rows x 128 B
+constexpr uint32_t kQBytes = 2 * kHalf;                // Q: two head-dim halves
+constexpr uint32_t kStageBytes = 4 * kHalf;            // K0 K1 V0 V1
+constexpr uint32_t kOffStages = kQBytes;
+constexpr uint32_t kOffCtrl = kOffStages + kStagesTC * kStageBytes;
+
+constexpr uint32_t kIdescS = idesc_bf16_f32(128, kN, 0, 0);     // K-major A and B
+constexpr uint32_t kIdescPV = idesc_bf16_f32(128, kD, 0, 1);    // B (V) MN-major
+
+struct TileMeta {
+  int32_t unit;        // < 0: no more tiles
+  int32_t b, g;
+  int32_t tile;        // tile index within the sequence
+  int32_t first, last; // first / last tile of the unit
+  int32_t nq, nd;      // query positions; draft rows (draft mode)
+  int32_t ncp;         // cache pages of the sequence
+  int32_t cvalid;      // cache rows that exist (L, or L + n_q for verify)
+  int32_t lim0;        // query j sees cache positions <= lim0 + j
+  int32_t rec0;        // first partial record of the (b, g) pair
+  int32_t chunk;       // unit index within the pair
+  int32_t nunits;      // units of the pair
+  int32_t pad[2];
+};
+
+struct Ctrl {
+  uint64_t kv_full[kStagesTC];
+  uint64_t kv_empty[kStagesTC];
+  uint64_t q_full, q_empty;
+  uint64_t s_full[2], p_full[2];
+  uint64_t o_full;
+  uint32_t tmem_base;
+  volatile int32_t abort_flag;
+  TileMeta meta[kStagesTC];
+};
+
+constexpr size_t kSmemTC = kOffCtrl + sizeof(Ctrl) + 1024;   // + alignment slack
+static_assert(kSmemTC <= 232448, "shared memory budget");
+
+__device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, Ctrl* c,
+                                              int32_t* err) {
+  for (uint32_t i = 0; i < kSpinLimit; ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (c->abort_flag) return false;
+    if (i >= 32) __nanosleep(64);
+  }
+  c->abort_flag = 1;
+  raise_err(err, SEED_DEVERR_TIMEOUT);
+  return false;
+}
+
+// ------------------------------------------------------------- sequences
+struct SeqT {
+  int nq, nd, ncp, cvalid, lim0, tiles, bad;
+};
+
+__device__ __forceinline__ SeqT seq_of(const AttnTcParams& p, int b) {
+  SeqT s{};
+  const int L = p.ctx_lens[b];
+  const int a = p.aux[b];
+  const long long cap = (long long)p.max_pages * kPage;
+  if (p.draft) {
+    if (a < 0 || a > p.kmax) s.bad |= SEED_DEVERR_DRAFT_LEN;
+    if (L < 0 || (long long)L > cap) s.bad |= SEED_DEVERR_CTX_LEN;
+    if (s.bad || a == 0) return s;
+    s.nq = 1;
+    s.nd = a;
+    s.cvalid = L;
+    s.lim0 = L - 1;
+    s.ncp = (L + kPage - 1) / kPage;
+    s.tiles = (s.ncp + 1 + kPagesPerTile - 1) / kPagesPerTile;
+  } else {
+    if (a < 0 || a > p.kmax + 1) s.bad |= SEED_DEVERR_NQ;
+    if (L < 0 || (long long)L + a > cap) s.bad |= SEED_DEVERR_CTX_LEN;
+    if (s.bad || a == 0) return s;
+    s.nq = a;
+    s.cvalid = L + a;
+    s.lim0 = L;
+    s.ncp = (s.cvalid + kPage - 1) / kPage;
+    s.tiles = (s.ncp + kPagesPerTile - 1) / kPagesPerTile;
+  }
+  return s;
+}
+
+struct Plan {
+  int tpu, full_total, units;
+};
+
+__device__ Plan make_plan(const AttnTcParams& p, int lane) {
+  long long tot = 0;
+  for (int b = lane; b < p.B; b += 32) tot += seq_of(p, b).tiles;
+  for (int o = 16; o; o >>= 1) tot += __shfl_xor_sync(kFull, tot, o);
+  tot *= p.hkv;
+  Plan pl;
+  pl.tpu = (int)max(1LL, (tot + p.target_units - 1) / p.target_units);
+  int full = 0, part = 0;
+  for (int b = lane; b < p.B; b += 32) {
+    const int t = seq_of(p, b).tiles;
+    full += p.hkv * (t / pl.tpu);
+    part += p.hkv * ((t % pl.tpu) != 0);
+  }
+  for (int o = 16; o; o >>= 1) {
+    full += __shfl_xor_sync(kFull, full, o);
+    part += __shfl_xor_sync(kFull, part, o);
+  }
+  pl.full_total = full;
+  pl.units = full + part;
+  return pl;
+}
+
+struct UnitInfo {
+  int b, g, chunk, t0, t1, rec0, nunits;
+  SeqT s;
+};
+
+// Warp-cooperative: map dense unit index u to (b, g, chunk).  Units
+// [0, full_total) are the full-size units (tpu tiles) of all pairs, the rest
+// the ragged last units.  Record indices follow (b, g, chunk) order.
+__device__ UnitInfo lookup_unit(const AttnTcParams& p, const Plan& pl, int u, int lane) {
+  const bool full_phase = u < pl.full_total;
+  const int target = full_phase ? u : u - pl.full_total;
+  int base1 = 0, base2 = 0;
+  UnitInfo ui{};
+  ui.b = -1;
+  for (int start = 0; start < p.B; start += 32) {
+    const int b = start + lane;
+    int a1 = 0, a2 = 0;
+    SeqT st{};
+    if (b < p.B) {
+      st = seq_of(p, b);
+      const int F = st.tiles / pl.tpu, P = (st.tiles % pl.tpu) != 0;
+      a1 = p.hkv * (full_phase ? F : P);
+      a2 = p.hkv * (F + P);
+    }
+    int s1 = a1, s2 = a2;
+    for (int o = 1; o < 32; o <<= 1) {
+      const int t1 = __shfl_up_sync(kFull, s1, o), t2 = __shfl_up_sync(kFull, s2, o);
+      if (lane >= o) {
+        s1 += t1;
+        s2 += t2;
+      }
+    }
+    const bool hit = b < p.B && a1 > 0 && base1 + s1 - a1 <= target && target < base1 + s1;
+    const unsigned m = __ballot_sync(kFull, hit);
+    if (m) {
+      const int src = __ffs(m) - 1;
+      const int pre1 = base1 + __shfl_sync(kFull, s1 - a1, src);
+      const int pre2 = base2 + __shfl_sync(kFull, s2 - a2, src);
+      ui.b = start + src;
+      ui.s.nq = __shfl_sync(kFull, st.nq, src);
+      ui.s.nd = __shfl_sync(kFull, st.nd, src);
+      ui.s.ncp = __shfl_sync(kFull, st.ncp, src);
+      ui.s.cvalid = __shfl_sync(kFull, st.cvalid, src);
+      ui.s.lim0 = __shfl_sync(kFull, st.lim0, src);
+      ui.s.tiles = __shfl_sync(kFull, st.tiles, src);
+      const int F = ui.s.tiles / pl.tpu, P = (ui.s.tiles % pl.tpu) != 0;
+      ui.nunits = F + P;
+      const int r = target - pre1;
+      if (full_phase) {
+        ui.g = r / F;
+        ui.chunk = r - ui.g * F;
+        ui.t0 = ui.chunk * pl.tpu;
+        ui.t1 = ui.t0 + pl.tpu;
+      } else {
+        ui.g = r;
+        ui.chunk = F;
+        ui.t0 = F * pl.tpu;
+        ui.t1 = ui.s.tiles;
+      }
+      ui.rec0 = pre2 + ui.g * ui.nunits;
+      return ui;
+    }
+    base1 += __shfl_sync(kFull, s1, 31);
+    base2 += __shfl_sync(kFull, s2, 31);
+  }
+  return ui;
+}
+
+// ------------------------------------------------------------- the kernel
+__global__ void __launch_bounds__(kThreadsTC, 1)
+    attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
+                   const __grid_constant__ CUtensorMap tm_k,
+                   const __grid_constant__ CUtensorMap tm_v,
+                   const __grid_constant__ CUtensorMap tm_dk,
+                   const __grid_constant__ CUtensorMap tm_dv, const AttnTcParams p) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  // the 128-byte swizzled tiles need a 1 KiB aligned base
+  uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+  Ctrl* ctrl = reinterpret_cast<Ctrl*>(smem + kOffCtrl);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const uint32_t sbase = smem_u32(smem);
+
+  if (tid == 0) {
+    for (int s = 0; s < kStagesTC; ++s) {
+      mbar_init(&ctrl->kv_full[s], 1);
+      mbar_init(&ctrl->kv_empty[s], 1);
+    }
+    mbar_init(&ctrl->q_full, 1);
+    mbar_init(&ctrl->q_empty, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&ctrl->s_full[i], 1);
+      mbar_init(&ctrl->p_full[i], 4);
+    }
+    mbar_init(&ctrl->o_full, 1);
+    ctrl->abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(&ctrl->tmem_base, kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = ctrl->tmem_base;
+  const int Rmax = p.G * p.W1;
+
+  if (warp == 0) {
+    // ---------------------------------------------------------- producer
+    if (lane == 0) {
+      tma_prefetch_desc(&tm_q);
+      tma_prefetch_desc(&tm_k);
+      tma_prefetch_desc(&tm_v);
+      if (p.draft) {
+        tma_prefetch_desc(&tm_dk);
+        tma_prefetch_desc(&tm_dv);
+      }
+    }
+    const Plan pl = make_plan(p, lane);
+    if (blockIdx.x == 0) {
+      for (int b = lane; b < p.B; b += 32) {
+        const int bad = seq_of(p, b).bad;
+        if (bad) raise_err(p.err, bad);
+      }
+    }
+    int it = 0, uo = 0;
+    bool ok = true;
+    while (ok) {
+      int u = 0;
+      if (lane == 0) u = atomicAdd(&p.sched[0], 1);
+      u = __shfl_sync(kFull, u, 0);
+      if (u >= pl.units) break;
+      const UnitInfo ui = lookup_unit(p, pl, u, lane);
+      if (ui.b < 0) break;
+      for (int t = ui.t0; t < ui.t1 && ok; ++t, ++it) {
+        const int s = it % kStagesTC;
+        // page ids of this tile, one lane per page
+        const int vp = t * kPagesPerTile + (lane & 7);
+        int pid = -1;
+        if (lane < kPagesPerTile && vp < ui.s.ncp) {
+          pid = p.page_table[(size_t)ui.b * p.max_pages + vp];
+          if (pid < 0 || pid >= p.num_pages) {
+            raise_err(p.err, SEED_DEVERR_PAGE);
+            pid = -1;
+          }
+        }
+        if (it >= kStagesTC)
+          ok = wait_or_abort(&ctrl->kv_empty[s], ((it / kStagesTC) - 1) & 1, ctrl, p.err);
+        if (ok && t == ui.t0 && uo > 0) ok = wait_or_abort(&ctrl->q_empty, (uo - 1) & 1, ctrl, p.err);
+        if (!ok) break;
+        int pids[kPagesPerTile];
+#pragma unroll
+        for (int pp = 0; pp < kPagesPerTile; ++pp) pids[pp] = __shfl_sync(kFull, pid, pp);
+        if (lane == 0) {
+          TileMeta& m = ctrl->meta[s];
+          m.unit = u;
+          m.b = ui.b;
+          m.g = ui.g;
+          m.tile = t;
+          m.first = (t == ui.t0);
+          m.last = (t == ui.t1 - 1);
+          m.nq = ui.s.nq;
+          m.nd = ui.s.nd;
+          m.ncp = ui.s.ncp;
+          m.cvalid = ui.s.cvalid;
+          m.lim0 = ui.s.lim0;
+          m.rec0 = ui.rec0;
+          m.chunk = ui.chunk;
+          m.nunits = ui.nunits;
+          if (t == ui.t0) {
+            mbar_arrive_expect_tx(&ctrl->q_full, 2u * 128u * (uint32_t)Rmax);
+            tma_load_4d(smem, &tm_q, 0, ui.g * p.G, 0, ui.b, &ctrl->q_full);
+            tma_load_4d(smem + kHalf, &tm_q, 64, ui.g * p.G, 0, ui.b, &ctrl->q_full);
+          }
+          const int dslot = ui.s.nd > 0 ? ui.s.ncp - t * kPagesPerTile : -1;   // draft page slot
+          uint32_t bytes = 0;
+#pragma unroll
+          for (int pp = 0; pp < kPagesPerTile; ++pp)
+            if (pids[pp] >= 0 || pp == dslot) bytes += 4u * 2048u;
+          mbar_arrive_expect_tx(&ctrl->kv_full[s], bytes);
+          uint8_t* st = smem + kOffStages + (size_t)s * kStageBytes;
+#pragma unroll
+          for (int pp = 0; pp < kPagesPerTile; ++pp) {
+            const uint32_t off = pp * 2048u;
+            if (pids[pp] >= 0) {
+              tma_load_4d(st + 0 * kHalf + off, &tm_k, 0, 0, ui.g, pids[pp], &ctrl->kv_full[s]);
+              tma_load_4d(st + 1 * kHalf + off, &tm_k, 64, 0, ui.g, pids[pp], &ctrl->kv_full[s]);
+              tma_load_4d(st + 2 * kHalf + off, &tm_v, 0, 0, ui.g, pids[pp], &ctrl->kv_full[s]);
+              tma_load_4d(st + 3 * kHalf + off, &tm_v, 64, 0, ui.g, pids[pp], &ctrl->kv_full[s]);
+            } else if (pp == dslot) {
+              tma_load_4d(st + 0 * kHalf + off, &tm_dk, 0, 0, ui.g, ui.b, &ctrl->kv_full[s]);
+              tma_load_4d(st + 1 * kHalf + off, &tm_dk, 64, 0, ui.g, ui.b, &ctrl->kv_full[s]);
+              tma_load_4d(st + 2 * kHalf + off, &tm_dv, 0, 0, ui.g, ui.b, &ctrl->kv_full[s]);
+              tma_load_4d(st + 3 * kHalf + off, &tm_dv, 64, 0, ui.g, ui.b, &ctrl->kv_full[s]);
+            }
+          }
+        }
+        __syncwarp();
+      }
+      ++uo;
+    }
+    // end marker for the consumers
+    if (ok) {
+      const int s = it % kStagesTC;
+      if (it >= kStagesTC) ok = wait_or_abort(&ctrl->kv_empty[s], ((it / kStagesTC) - 1) & 1, ctrl, p.err);
+      if (ok && lane == 0) {
+        ctrl->meta[s].unit = -1;
+        mbar_arrive(&ctrl->kv_full[s]);
+      }
+    }
+  } else if (warp == 1) {
+    // ---------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      int t = 0, uo = 0;
+      int prev_first = 0;
+      bool have_prev = false;
+      while (true) {
+        const int s = t % kStagesTC;
+        if (!wait_or_abort(&ctrl->kv_full[s], (t / kStagesTC) & 1, ctrl, p.err)) break;
+        const int unit = ctrl->meta[s].unit;
+        const int first = ctrl->meta[s].first, last = ctrl->meta[s].last;
+        if (unit >= 0) {
+          if (first) {
+            if (!wait_or_abort(&ctrl->q_full, uo & 1, ctrl, p.err)) break;
+            ++uo;
+          }
+          if (t >= 2 && !wait_or_abort(&ctrl->o_full, (t - 2) & 1, ctrl, p.err)) break;
+          tc_fence_after();
+          const uint32_t d = tmem + (uint32_t)(t & 1) * kN;
+          const uint32_t kb = sbase + kOffStages + (uint32_t)s * kStageBytes;
+#pragma unroll
+          for (int kk = 0; kk < kD / 16; ++kk) {
+            const uint32_t h = kk >> 2, off = (kk & 3) * 32;
+            const uint64_t a = smem_desc_sw128(sbase + h * kHalf + off, 16, 1024);
+            const uint64_t b = smem_desc_sw128(kb + h * kHalf + off, 16, 1024);
+            mma_ss(d, a, b, kIdescS, kk > 0);
+          }
+          mma_commit(&ctrl->s_full[t & 1]);
+          if (last) mma_commit(&ctrl->q_empty);
+        }
+        if (have_prev) {
+          const int tp = t - 1;
+          if (!wait_or_abort(&ctrl->p_full[tp & 1], (tp >> 1) & 1, ctrl, p.err)) break;
+          tc_fence_after();
+          const int sp = tp % kStagesTC;
+          const uint32_t pcol = tmem + (uint32_t)(tp & 1) * kN;
+          const uint32_t vb = sbase + kOffStages + (uint32_t)sp * kStageBytes + 2 * kHalf;
+#pragma unroll
+          for (int kk = 0; kk < kN / 16; ++kk) {
+            const uint64_t b = smem_desc_sw128(vb + kk * 2048u, kHalf, 1024);
+            mma_ts(tmem + kColO, pcol + kk * 8, b, kIdescPV, !(prev_first && kk == 0));
+          }
+#pragma unroll
+          for (int kk = 0; kk < kN / 16; ++kk) {
+            const uint64_t b = smem_desc_sw128(vb + kk * 2048u, kHalf, 1024);
+            mma_ts(tmem + kColO, pcol + 64 + kk * 8, b, kIdescPV, 1);
+          }
+          mma_commit(&ctrl->o_full);
+          mma_commit(&ctrl->kv_empty[sp]);
+        }
+        if (unit < 0) break;
+        prev_first = first;
+        have_prev = true;
+        ++t;
+      }
+    }
+    __syncwarp();
+  } else {
+    // ---------------------------------------------------------- softmax
+    const int q4 = warp & 3;                  // TMEM lane quarter of this warp
+    const int row = q4 * 32 + lane;           // query row = j * G + head in group
+    const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
+    const int col = tid - 64;                 // 0..127: the column this thread zeroes
+    float m_used = -INFINITY, l = 0.f;
+    int t = 0;
+    while (!ctrl->abort_flag) {
+      const int s = t % kStagesTC;
+      if (!wait_or_abort(&ctrl->kv_full[s], (t / kStagesTC) & 1, ctrl, p.err)) break;
+      const TileMeta m = ctrl->meta[s];
+      if (m.unit < 0) break;
+      if (!wait_or_abort(&ctrl->s_full[t & 1], (t >> 1) & 1, ctrl, p.err)) break;
+      tc_fence_after();
+      if (m.first) {
+        m_used = -INFINITY;
+        l = 0.f;
+      }
+      const int R = m.nq * p.G;
+      const int j = row / p.G;
+      const bool warp_active = q4 * 32 < R;
+      const int dcol = (m.ncp - m.tile * kPagesPerTile) * kPage;   // first draft column
+      const int dend = dcol + m.nd;
+      bool resc = false;
+      float fo = 1.f;
+      const uint32_t scol = tmem + lane_off + (uint32_t)(t & 1) * kN;
+      if (warp_active) {
+        float x[kN];
+        {
+          uint32_t r0[32], r1[32], r2[32], r3[32];
+          tmem_ld32(scol + 0, r0);
+          tmem_ld32(scol + 32, r1);
+          tmem_ld32(scol + 64, r2);
+          tmem_ld32(scol + 96, r3);
+          tmem_wait_ld();
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            x[i] = __uint_as_float(r0[i]);
+            x[32 + i] = __uint_as_float(r1[i]);
+            x[64 + i] = __uint_as_float(r2[i]);
+            x[96 + i] = __uint_as_float(r3[i]);
+          }
+        }
+        const int lim = m.lim0 + j - m.tile * kN;     // cache columns c <= lim are visible
+        float mt = -INFINITY;
+#pragma unroll
+        for (int c = 0; c < kN; ++c) {
+          const bool vis = (c < dcol) ? (c <= lim) : (c < dend);
+          x[c] = vis ? x[c] * p.scale_log2 : -INFINITY;
+          mt = fmaxf(mt, x[c]);
+        }
+        if (mt > m_used + kRescale) {
+          const float f = (m_used == -INFINITY) ? 0.f : exp2f(m_used - mt);
+          if (!m.first && m_used != -INFINITY) {
+            resc = true;
+            fo = f;
+          }
+          l *= f;
+          m_used = mt;
+        }
+        const float mu = (m_used == -INFINITY) ? 0.f : m_used;
+        float lsum = 0.f;
+        // P_hi of tokens [64h, 64h+64) -> packed columns [32h, 32h+32),
+        // P_lo -> [64 + 32h, 64 + 32h + 32); even token in the low half-word
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+          uint32_t wh[32], wl[32];
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const float p0 = exp2f(x[64 * half + 2 * i] - mu);
+            const float p1 = exp2f(x[64 * half + 2 * i + 1] - mu);
+            lsum += p0 + p1;
+            const uint32_t h = pack_bf16x2(p0, p1);
+            wh[i] = h;
+            wl[i] = pack_bf16x2(p0 - bf16lo(h), p1 - bf16hi(h));
+          }
+          tmem_st32(scol + 32 * half, wh);
+          tmem_st32(scol + 64 + 32 * half, wl);
+        }
+        tmem_wait_st();
+        l += lsum;
+      }
+      // V rows of columns nobody may see are zeroed, so that a probability of
+      // 0 never meets a stale or NaN-poisoned row
+      {
+        const bool valid = (col < dcol) ? (col < m.cvalid - m.tile * kN) : (col < dend);
+        if (!valid) {
+          uint8_t* vb = smem + kOffStages + (size_t)s * kStageBytes + 2 * kHalf;
+#pragma unroll
+          for (int ch = 0; ch < 8; ++ch) {
+            *reinterpret_cast<uint4*>(vb + col * 128 + ch * 16) = make_uint4(0, 0, 0, 0);
+            *reinterpret_cast<uint4*>(vb + kHalf + col * 128 + ch * 16) = make_uint4(0, 0, 0, 0);
+          }
+          fence_proxy_async_smem();
+        }
+      }
+      // the previous PV must be done before O is rescaled (and before the
+      // next one is issued on top of it)
+      if (t > 0 && !wait_or_abort(&ctrl->o_full, (t - 1) & 1, ctrl, p.err)) break;
+      tc_fence_after();
+      if (warp_active && __any_sync(kFull, resc)) {
+        const float f = resc ? fo : 1.f;
+        uint32_t r0[32], r1[32], r2[32], r3[32];
+        tmem_ld32(tmem + lane_off + kColO + 0, r0);
+        tmem_ld32(tmem + lane_off + kColO + 32, r1);
+        tmem_ld32(tmem + lane_off + kColO + 64, r2);
+        tmem_ld32(tmem + lane_off + kColO + 96, r3);
+        tmem_wait_ld();
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          r0[i] = __float_as_uint(__uint_as_float(r0[i]) * f);
+          r1[i] = __float_as_uint(__uint_as_float(r1[i]) * f);
+          r2[i] = __float_as_uint(__uint_as_float(r2[i]) * f);
+          r3[i] = __float_as_uint(__uint_as_float(r3[i]) * f);
+        }
+        tmem_st32(tmem + lane_off + kColO + 0, r0);
+        tmem_st32(tmem + lane_off + kColO + 32, r1);
+        tmem_st32(tmem + lane_off + kColO + 64, r2);
+        tmem_st32(tmem + lane_off + kColO + 96, r3);
+        tmem_wait_st();
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctrl->p_full[t & 1]);
+
+      if (m.last) {
+        // ------------------------------------------------------ epilogue
+        if (!wait_or_abort(&ctrl->o_full, t & 1, ctrl, p.err)) break;
+        tc_fence_after();
+        if (warp_active) {
+          const int REC = Rmax * (kD + 1);
+          const bool real = row < R;
+          const int qh = m.g * p.G + (row - j * p.G);
+          const size_t orow = ((size_t)m.b * p.W1 + j) * p.hq + qh;   // [b, j, head]
+          const float inv = (l > 0.f) ? 1.f / l : 0.f;
+          const float lse2 = (l > 0.f) ? m_used + log2f(l) : -INFINITY;
+          uint32_t r0[32], r1[32], r2[32], r3[32];
+          tmem_ld32(tmem + lane_off + kColO + 0, r0);
+          tmem_ld32(tmem + lane_off + kColO + 32, r1);
+          tmem_ld32(tmem + lane_off + kColO + 64, r2);
+          tmem_ld32(tmem + lane_off + kColO + 96, r3);
+          tmem_wait_ld();
+          if (m.nunits == 1) {
+            if (real) {
+              float* dst = p.out + orow * kD;
+#pragma unroll
+              for (int i = 0; i < 32; i += 4) {
+                *reinterpret_cast<float4*>(dst + i) =
+                    make_float4(__uint_as_float(r0[i]) * inv, __uint_as_float(r0[i + 1]) * inv,
+                                __uint_as_float(r0[i + 2]) * inv, __uint_as_float(r0[i + 3]) * inv);
+                *reinterpret_cast<float4*>(dst + 32 + i) =
+                    make_float4(__uint_as_float(r1[i]) * inv, __uint_as_float(r1[i + 1]) * inv,
+                                __uint_as_float(r1[i + 2]) * inv, __uint_as_float(r1[i + 3]) * inv);
+                *reinterpret_cast<float4*>(dst + 64 + i) =
+                    make_float4(__uint_as_float(r2[i]) * inv, __uint_as_float(r2[i + 1]) * inv,
+                                __uint_as_float(r2[i + 2]) * inv, __uint_as_float(r2[i + 3]) * inv);
+                *reinterpret_cast<float4*>(dst + 96 + i) =
+                    make_float4(__uint_as_float(r3[i]) * inv, __uint_as_float(r3[i + 1]) * inv,
+                                __uint_as_float(r3[i + 2]) * inv, __uint_as_float(r3[i + 3]) * inv);
+              }
+              if (p.lse != nullptr) p.lse[orow] = lse2 * kLn2;
+            }
+          } else {
+            // partial record, column-major [d][row] so that the rows of a warp
+            // store (and later load) contiguously
+            float* rec = p.part + (size_t)(m.rec0 + m.chunk) * REC;
+            if (real) {
+#pragma unroll
+              for (int i = 0; i < 32; ++i) {
+                rec[(size_t)i * Rmax + row] = __uint_as_float(r0[i]) * inv;
+                rec[(size_t)(32 + i) * Rmax + row] = __uint_as_float(r1[i]) * inv;
+                rec[(size_t)(64 + i) * Rmax + row] = __uint_as_float(r2[i]) * inv;
+                rec[(size_t)(96 + i) * Rmax + row] = __uint_as_float(r3[i]) * inv;
+              }
+              rec[(size_t)kD * Rmax + row] = lse2;
+            }
+            __threadfence();
+            __syncwarp();
+            int last = 0;
+            if (lane == 0)
+              last = atomicAdd(&p.counters[(m.b * p.hkv + m.g) * 4 + q4], 1) == m.nunits - 1;
+            last = __shfl_sync(kFull, last, 0);
+            if (last) {
+              // this warp merges its rows over all units of the pair
+              __threadfence();
+              if (real) {
+                const float* base = p.part + (size_t)m.rec0 * REC;
+                float M = -INFINITY;
+                for (int c = 0; c < m.nunits; ++c)
+                  M = fmaxf(M, __ldcg(base + (size_t)c * REC + (size_t)kD * Rmax + row));
+                float S = 0.f;
+                for (int c = 0; c < m.nunits; ++c) {
+                  const float lc = __ldcg(base + (size_t)c * REC + (size_t)kD * Rmax + row);
+                  S += (lc == -INFINITY) ? 0.f : exp2f(lc - M);
+                }
+                const float invS = 1.f / S;
+                float* dst = p.out + orow * kD;
+#pragma unroll 1
+                for (int d0 = 0; d0 < kD; d0 += 32) {
+                  float acc[32];
+#pragma unroll
+                  for (int i = 0; i < 32; ++i) acc[i] = 0.f;
+                  for (int c = 0; c < m.nunits; ++c) {
+                    const float* rc = base + (size_t)c * REC;
+                    const float lc = __ldcg(rc + (size_t)kD * Rmax + row);
+                    const float w = (lc == -INFINITY) ? 0.f : exp2f(lc - M) * invS;
+#pragma unroll
+                    for (int i = 0; i < 32; ++i)
+                      acc[i] = fmaf(w, __ldcg(rc + (size_t)(d0 + i) * Rmax + row), acc[i]);
+                  }
+#pragma unroll
+                  for (int i = 0; i < 32; i += 4)
+                    *reinterpret_cast<float4*>(dst + d0 + i) =
+                        make_float4(acc[i], acc[i + 1], acc[i + 2], acc[i + 3]);
+                }
+                if (p.lse != nullptr) p.lse[orow] = (M + log2f(S)) * kLn2;
+              }
+              if (lane == 0) p.counters[(m.b * p.hkv + m.g) * 4 + q4] = 0;
+            }
+          }
+        }
+      }
+      ++t;
+    }
+  }
+
+  // ------------------------------------------------------------ teardown
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+  if (tid == 0) {
+    __threadfence();
+    if (atomicAdd(&p.sched[1], 1) == (int)gridDim.x - 1) {
+      p.sched[0] = 0;
+      p.sched[1] = 0;
+      __threadfence();
+    }
+  }
+}
+
+// ------------------------------------------------------------- host side
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(ptr);
+  });
+  return fn;
+}
+
+// 4-d bf16 tensor map, innermost dimension = 128 head dims, 128-byte swizzle.
+bool encode_4d(CUtensorMap* map, const void* base, const cuuint64_t dims[4],
+               const cuuint64_t strides[3], const cuuint32_t box[4]) {
+  EncodeTiledFn fn = encode_fn();
+  if (fn == nullptr) return false;
+  const cuuint32_t elem[4] = {1, 1, 1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box,
+            elem, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+std::atomic<uint64_t> g_tc_attr_set{0};
+
+}  // namespace
+
+bool attn_tc_supported(int head_dim, int group, int w1) {
+  return head_dim == kD && group * w1 <= 128;
+}
+
+int attn_tc_target_units() { return std::min(2 * device_sm_count(), kTcUnitsCap); }
+
+cudaError_t launch_attn_tc(const AttnTcParams& prm, const void* q, const void* k_cache,
+                           const void* v_cache, const void* draft_k, const void* draft_v,
+                           cudaStream_t st) {
+  CUtensorMap tq, tk, tv, tdk, tdv;
+  const uint64_t W1 = (uint64_t)prm.W1;
+  {
+    const cuuint64_t dims[4] = {kD, (cuuint64_t)prm.hq, W1, (cuuint64_t)prm.B};
+    const cuuint64_t strides[3] = {kD * 2ull, (cuuint64_t)prm.hq * kD * 2ull,
+                                   W1 * prm.hq * kD * 2ull};
+    const cuuint32_t box[4] = {64, (cuuint32_t)prm.G, (cuuint32_t)W1, 1};
+    if (!encode_4d(&tq, q, dims, strides, box)) return cudaErrorInvalidValue;
+  }
+  {
+    const cuuint64_t dims[4] = {kD, (cuuint64_t)kPage, (cuuint64_t)prm.hkv,
+                                (cuuint64_t)prm.num_pages};
+    const cuuint64_t strides[3] = {kD * 2ull, kPage * kD * 2ull,
+                                   (cuuint64_t)prm.hkv * kPage * kD * 2ull};
+    const cuuint32_t box[4] = {64, (cuuint32_t)kPage, 1, 1};
+    if (!encode_4d(&tk, k_cache, dims, strides, box)) return cudaErrorInvalidValue;
+    if (!encode_4d(&tv, v_cache, dims, strides, box)) return cudaErrorInvalidValue;
+  }
+  if (prm.draft) {
+    // draft scratch [B, hkv, kmax, D]: one box = the 16-row draft page (rows
+    // past kmax are filled with zeros by the copy engine)
+    const cuuint64_t dims[4] = {kD, (cuuint64_t)prm.kmax, (cuuint64_t)prm.hkv, (cuuint64_t)prm.B};
+    const cuuint64_t strides[3] = {kD * 2ull, (cuuint64_t)prm.kmax * kD * 2ull,
+                                   (cuuint64_t)prm.hkv * prm.kmax * kD * 2ull};
+    const cuuint32_t box[4] = {64, (cuuint32_t)kPage, 1, 1};
+    if (!encode_4d(&tdk, draft_k, dims, strides, box)) return cudaErrorInvalidValue;
+    if (!encode_4d(&tdv, draft_v, dims, strides, box)) return cudaErrorInvalidValue;
+  } else {
+    tdk = tk;
+    tdv = tv;
+  }
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const uint64_t bit = 1ull << (dev & 63);
+  if (!(g_tc_attr_set.load(std::memory_order_acquire) & bit)) {
+    e = cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)kSmemTC);
+    if (e != cudaSuccess) return e;
+    g_tc_attr_set.fetch_or(bit, std::memory_order_acq_rel);
+  }
+  const int grid = device_sm_count();
+  attn_tc_kernel<<<grid, kThreadsTC, kSmemTC, st>>>(tq, tk, tv, tdk, tdv, prm);
+  return cudaGetLastError();
+}
+
+size_t attn_tc_part_bound(int32_t batch, int32_t hkv, int32_t group, int32_t w1) {
+  const size_t rmax = (size_t)group * w1;
+  return ((size_t)kTcUnitsCap + (size_t)batch * hkv) * rmax * (kD + 1) * sizeof(float);
+}
+
+}  // namespace seedk

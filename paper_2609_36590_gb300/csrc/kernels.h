@@ -69,30 +69,33 @@ cudaError_t launch_accept(int32_t B, int32_t kmax, const int32_t* draft_ids,
 
 int device_sm_count();
 
-// Tensor-core verify attention (verify_tc.cu).
-constexpr int kTcUnitsCap = 1024;   // most work units one verify launch plans
+// Tensor-core draft and verify attention (attn_tc.cu).
+constexpr int kTcUnitsCap = 1024;   // most work units one launch plans
 
-struct VerifyTcParams {
+struct AttnTcParams {
   const int32_t* page_table;
   int32_t max_pages;
   int32_t num_pages;
   const int32_t* ctx_lens;    // [B]
-  const int32_t* n_q;         // [B]
-  float* out;                 // f32 [B, kmax+1, hq, 128]
-  float* lse;                 // f32 [B, kmax+1, hq] or null
+  const int32_t* aux;         // verify: n_q [B]; draft: draft_lens [B]
+  float* out;                 // f32 [B, W1, hq, 128]
+  float* lse;                 // f32 [B, W1, hq] or null
   float* part;                // partial records
-  int32_t* counters;          // [B * hkv] arrival counters (zero between calls)
+  int32_t* counters;          // [B * hkv * 4] arrival counters (zero between calls)
   int32_t* sched;             // [2] unit dispenser and finished-CTA count (zero between calls)
   int32_t* err;
   int32_t B, hq, hkv, kmax, G;
+  int32_t draft;              // 1: draft attention (cache rows + draft scratch rows)
+  int32_t W1;                 // query positions per sequence: kmax+1 (verify) or 1 (draft)
   int32_t target_units;
   float scale_log2;
 };
 
-bool verify_tc_supported(int head_dim, int group, int kmax);
-int verify_tc_target_units();
-size_t verify_tc_part_bound(int32_t batch, int32_t hkv, int32_t group, int32_t kmax);
-cudaError_t launch_verify_tc(const VerifyTcParams& p, const void* q, const void* k_cache,
-                             const void* v_cache, cudaStream_t st);
+bool attn_tc_supported(int head_dim, int group, int w1);
+int attn_tc_target_units();
+size_t attn_tc_part_bound(int32_t batch, int32_t hkv, int32_t group, int32_t w1);
+cudaError_t launch_attn_tc(const AttnTcParams& p, const void* q, const void* k_cache,
+                           const void* v_cache, const void* draft_k, const void* draft_v,
+                           cudaStream_t st);
 
 }  // namespace seedk

@@ -45,7 +45,8 @@ float scale_of(const seed_cfg_t* cfg) {
 constexpr size_t kSchedBytes = kAlign;
 
 size_t counters_bytes(const seed_cfg_t* cfg, int32_t batch) {
-  return round_up((size_t)batch * (cfg->kmax + 1) * cfg->hkv * sizeof(int32_t), kAlign);
+  const size_t per = std::max(cfg->kmax + 1, 4);
+  return round_up((size_t)batch * per * cfg->hkv * sizeof(int32_t), kAlign);
 }
 
 seed_status_t finish(cudaError_t e) { return e == cudaSuccess ? SEED_OK : SEED_ERR_CUDA; }
@@ -89,24 +90,25 @@ seed_status_t run_decode(const seed_cfg_t* cfg, int32_t batch, bool verify, cons
   return finish(seedk::launch_decode(p, cfg->head_dim, G, static_cast<cudaStream_t>(stream)));
 }
 
-// Verify attention on the tensor cores (head_dim 128, all G*(kmax+1) query
-// rows of a KV head in one 128-row tile).
-seed_status_t run_verify_tc(const seed_cfg_t* cfg, int32_t batch, const void* q,
-                            const int32_t* n_q, const seed_kv_t& kv, const int32_t* ctx_lens,
-                            float* out, float* lse, void* ws, size_t ws_bytes, int32_t* err,
-                            void* stream) {
+// Draft / verify attention on the tensor cores (head_dim 128, all query rows
+// of a KV head in one 128-row tile).
+seed_status_t run_attn_tc(const seed_cfg_t* cfg, int32_t batch, bool draft, const void* q,
+                          const int32_t* aux, const seed_kv_t& kv, const void* draft_k,
+                          const void* draft_v, const int32_t* ctx_lens, float* out, float* lse,
+                          void* ws, size_t ws_bytes, int32_t* err, void* stream) {
   const int G = cfg->hq / cfg->hkv;
+  const int W1 = draft ? 1 : cfg->kmax + 1;
   const size_t cb = kSchedBytes + counters_bytes(cfg, batch);
-  const int target = seedk::verify_tc_target_units();
-  const size_t need = cb + ((size_t)target + (size_t)batch * cfg->hkv) * G * (cfg->kmax + 1) *
+  const int target = seedk::attn_tc_target_units();
+  const size_t need = cb + ((size_t)target + (size_t)batch * cfg->hkv) * G * W1 *
                                (cfg->head_dim + 1) * sizeof(float);
   if (ws_bytes < need) return SEED_ERR_WORKSPACE;
-  seedk::VerifyTcParams p{};
+  seedk::AttnTcParams p{};
   p.page_table = kv.page_table;
   p.max_pages = kv.max_pages;
   p.num_pages = kv.num_pages;
   p.ctx_lens = ctx_lens;
-  p.n_q = n_q;
+  p.aux = aux;
   p.out = out;
   p.lse = lse;
   p.sched = static_cast<int32_t*>(ws);
@@ -118,9 +120,12 @@ seed_status_t run_verify_tc(const seed_cfg_t* cfg, int32_t batch, const void* q,
   p.hkv = cfg->hkv;
   p.kmax = cfg->kmax;
   p.G = G;
+  p.draft = draft ? 1 : 0;
+  p.W1 = W1;
   p.target_units = target;
   p.scale_log2 = scale_of(cfg) * 1.4426950408889634f;
-  return finish(seedk::launch_verify_tc(p, q, kv.k, kv.v, static_cast<cudaStream_t>(stream)));
+  return finish(seedk::launch_attn_tc(p, q, kv.k, kv.v, draft_k, draft_v,
+                                      static_cast<cudaStream_t>(stream)));
 }
 
 bool misaligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) != 0; }
@@ -149,8 +154,10 @@ size_t seed_workspace_bytes(const seed_cfg_t* cfg, int32_t batch) {
   const int G = cfg->hq / cfg->hkv;
   const int32_t nv_max = batch * (cfg->kmax + 1);
   size_t part = seedk::decode_workspace_bound(nv_max, cfg->hkv, G, cfg->head_dim);
-  if (seedk::verify_tc_supported(cfg->head_dim, G, cfg->kmax))
-    part = std::max(part, seedk::verify_tc_part_bound(batch, cfg->hkv, G, cfg->kmax));
+  if (seedk::attn_tc_supported(cfg->head_dim, G, 1))
+    part = std::max(part, seedk::attn_tc_part_bound(batch, cfg->hkv, G, 1));
+  if (seedk::attn_tc_supported(cfg->head_dim, G, cfg->kmax + 1))
+    part = std::max(part, seedk::attn_tc_part_bound(batch, cfg->hkv, G, cfg->kmax + 1));
   return kSchedBytes + counters_bytes(cfg, batch) + round_up(part, kAlign);
 }
 
@@ -186,6 +193,9 @@ seed_status_t seed_draft_attn(const seed_cfg_t* cfg, int32_t batch, const void* 
       misaligned16(draft_k) || misaligned16(draft_v))
     return SEED_ERR_RANGE;
   if ((reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)) != 0) return SEED_ERR_WORKSPACE;
+  if (seedk::attn_tc_supported(cfg->head_dim, cfg->hq / cfg->hkv, 1))
+    return run_attn_tc(cfg, batch, true, q, draft_lens, ctx_kv, draft_k, draft_v, ctx_lens, out,
+                       lse, ws, ws_bytes, err_flag, stream);
   return run_decode(cfg, batch, false, q, ctx_kv, draft_k, draft_v, ctx_lens, draft_lens, out, lse,
                     ws, ws_bytes, err_flag, stream);
 }
@@ -220,9 +230,9 @@ seed_status_t seed_verify_attn(const seed_cfg_t* cfg, int32_t batch, const void*
   if ((st = check_kv(kv)) != SEED_OK) return st;
   if (misaligned16(q) || misaligned16(kv.k) || misaligned16(kv.v)) return SEED_ERR_RANGE;
   if ((reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)) != 0) return SEED_ERR_WORKSPACE;
-  if (seedk::verify_tc_supported(cfg->head_dim, cfg->hq / cfg->hkv, cfg->kmax))
-    return run_verify_tc(cfg, batch, q, n_q, kv, ctx_lens, out, lse, ws, ws_bytes, err_flag,
-                         stream);
+  if (seedk::attn_tc_supported(cfg->head_dim, cfg->hq / cfg->hkv, cfg->kmax + 1))
+    return run_attn_tc(cfg, batch, false, q, n_q, kv, nullptr, nullptr, ctx_lens, out, lse, ws,
+                       ws_bytes, err_flag, stream);
   return run_decode(cfg, batch, true, q, kv, nullptr, nullptr, ctx_lens, n_q, out, lse, ws,
                     ws_bytes, err_flag, stream);
 }
