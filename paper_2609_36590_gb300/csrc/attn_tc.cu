@@ -31,9 +31,9 @@
 //
 // Work: units of `tpu` tiles of one (b, g) are handed out by an atomic
 // counter, full-size units first and ragged ones last.  Units of the same
-// (b, g) leave normalised partials and log2-sum-exps (column-major, so stores
-// and loads coalesce across the rows); per TMEM lane quarter the last warp to
-// finish merges them in unit order, so results are deterministic.
+// (b, g) leave normalised partials and log2-sum-exps; per TMEM lane quarter
+// the last warp to finish merges them in unit order, so results are
+// deterministic.
 //
 // Warp roles (192 threads): warp 0 TMA producer and scheduler, warp 1 MMA
 // issuer and TMEM owner, warps 2-5 softmax / epilogue.  Every wait is bounded;
@@ -56,9 +56,9 @@ constexpr int kD = 128;
 constexpr int kN = 128;                      // tokens (columns) per tile
 constexpr int kPagesPerTile = kN / kPage;    // 8
 constexpr int kStagesTC = 3;
-constexpr int kThreadsTC = 192;
+constexpr int kThreadsTC = 320;   // producer, MMA, 2 x 4 softmax warps
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColO = 256;              // O accumulator columns [256, 384)
+constexpr uint32_t kColO = 256;              // O accumulators: [256, 384) and [384, 512)
 constexpr float kRescale = 8.0f;
 constexpr float kLn2 = 0.69314718055994531f;
 constexpr unsigned kFull = 0xffffffffu;
@@ -76,7 +76,7 @@ struct TileMeta {
   int32_t unit;        // < 0: no more tiles
   int32_t b, g;
   int32_t tile;        // tile index within the sequence
-  int32_t first, last; // first / last tile of the unit
+  int32_t k, ntu;      // tile index within the unit; tiles in the unit
   int32_t nq, nd;      // query positions; draft rows (draft mode)
   int32_t ncp;         // cache pages of the sequence
   int32_t cvalid;      // cache rows that exist (L, or L + n_q for verify)
@@ -91,11 +91,12 @@ struct Ctrl {
   uint64_t kv_full[kStagesTC];
   uint64_t kv_empty[kStagesTC];
   uint64_t q_full, q_empty;
-  uint64_t s_full[2], p_full[2];
-  uint64_t o_full;
+  uint64_t s_full[2], p_full[2], o_full[2];   // per tile parity
+  uint64_t stats_bar[4], orel_bar[4];         // per TMEM lane quarter
   uint32_t tmem_base;
   volatile int32_t abort_flag;
   TileMeta meta[kStagesTC];
+  float xm[4][32], xl[4][32];                 // row statistics handed to the epilogue owner
 };
 
 constexpr size_t kSmemTC = kOffCtrl + sizeof(Ctrl) + 1024;   // + alignment slack
@@ -241,6 +242,12 @@ __device__ UnitInfo lookup_unit(const AttnTcParams& p, const Plan& pl, int u, in
 }
 
 // ------------------------------------------------------------- the kernel
+// One softmax row: the visible-column mask of tile `m` for query j.
+struct ColMask {
+  int dcol, dend, lim;
+  __device__ __forceinline__ bool vis(int c) const { return (c < dcol) ? (c <= lim) : (c < dend); }
+};
+
 __global__ void __launch_bounds__(kThreadsTC, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
                    const __grid_constant__ CUtensorMap tm_k,
@@ -264,8 +271,12 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     for (int i = 0; i < 2; ++i) {
       mbar_init(&ctrl->s_full[i], 1);
       mbar_init(&ctrl->p_full[i], 4);
+      mbar_init(&ctrl->o_full[i], 1);
     }
-    mbar_init(&ctrl->o_full, 1);
+    for (int i = 0; i < 4; ++i) {
+      mbar_init(&ctrl->stats_bar[i], 1);
+      mbar_init(&ctrl->orel_bar[i], 1);
+    }
     ctrl->abort_flag = 0;
     fence_mbar_init();
   }
@@ -331,8 +342,8 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
           m.b = ui.b;
           m.g = ui.g;
           m.tile = t;
-          m.first = (t == ui.t0);
-          m.last = (t == ui.t1 - 1);
+          m.k = t - ui.t0;
+          m.ntu = ui.t1 - ui.t0;
           m.nq = ui.s.nq;
           m.nd = ui.s.nd;
           m.ncp = ui.s.ncp;
@@ -373,8 +384,8 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
       }
       ++uo;
     }
-    // end marker for the consumers
-    if (ok) {
+    // end markers: one for each softmax parity (the MMA thread stops at the first)
+    for (int e = 0; e < 2 && ok; ++e, ++it) {
       const int s = it % kStagesTC;
       if (it >= kStagesTC) ok = wait_or_abort(&ctrl->kv_empty[s], ((it / kStagesTC) - 1) & 1, ctrl, p.err);
       if (ok && lane == 0) {
@@ -385,20 +396,21 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
   } else if (warp == 1) {
     // ---------------------------------------------------------- MMA issuer
     if (lane == 0) {
-      int t = 0, uo = 0;
-      int prev_first = 0;
+      int t = 0, uo = 0, prev_k = 0;
       bool have_prev = false;
       while (true) {
         const int s = t % kStagesTC;
         if (!wait_or_abort(&ctrl->kv_full[s], (t / kStagesTC) & 1, ctrl, p.err)) break;
         const int unit = ctrl->meta[s].unit;
-        const int first = ctrl->meta[s].first, last = ctrl->meta[s].last;
+        const int k = ctrl->meta[s].k;
+        const int last = ctrl->meta[s].k == ctrl->meta[s].ntu - 1;
         if (unit >= 0) {
-          if (first) {
+          if (k == 0) {
             if (!wait_or_abort(&ctrl->q_full, uo & 1, ctrl, p.err)) break;
             ++uo;
           }
-          if (t >= 2 && !wait_or_abort(&ctrl->o_full, (t - 2) & 1, ctrl, p.err)) break;
+          // S buffer t&1 is free once PV(t-2) has consumed its probabilities
+          if (t >= 2 && !wait_or_abort(&ctrl->o_full[t & 1], ((t - 2) >> 1) & 1, ctrl, p.err)) break;
           tc_fence_after();
           const uint32_t d = tmem + (uint32_t)(t & 1) * kN;
           const uint32_t kb = sbase + kOffStages + (uint32_t)s * kStageBytes;
@@ -418,22 +430,23 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
           tc_fence_after();
           const int sp = tp % kStagesTC;
           const uint32_t pcol = tmem + (uint32_t)(tp & 1) * kN;
+          const uint32_t ocol = tmem + kColO + (uint32_t)(tp & 1) * kD;
           const uint32_t vb = sbase + kOffStages + (uint32_t)sp * kStageBytes + 2 * kHalf;
 #pragma unroll
           for (int kk = 0; kk < kN / 16; ++kk) {
             const uint64_t b = smem_desc_sw128(vb + kk * 2048u, kHalf, 1024);
-            mma_ts(tmem + kColO, pcol + kk * 8, b, kIdescPV, !(prev_first && kk == 0));
+            mma_ts(ocol, pcol + kk * 8, b, kIdescPV, !(prev_k < 2 && kk == 0));
           }
 #pragma unroll
           for (int kk = 0; kk < kN / 16; ++kk) {
             const uint64_t b = smem_desc_sw128(vb + kk * 2048u, kHalf, 1024);
-            mma_ts(tmem + kColO, pcol + 64 + kk * 8, b, kIdescPV, 1);
+            mma_ts(ocol, pcol + 64 + kk * 8, b, kIdescPV, 1);
           }
-          mma_commit(&ctrl->o_full);
+          mma_commit(&ctrl->o_full[tp & 1]);
           mma_commit(&ctrl->kv_empty[sp]);
         }
         if (unit < 0) break;
-        prev_first = first;
+        prev_k = k;
         have_prev = true;
         ++t;
       }
@@ -441,91 +454,104 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
     __syncwarp();
   } else {
     // ---------------------------------------------------------- softmax
+    // Warps 2-5 take the even tiles of the CTA, warps 6-9 the odd ones; each
+    // group keeps its own running max, sum and O accumulator per row.
+    const int par = (warp - 2) >> 2;
     const int q4 = warp & 3;                  // TMEM lane quarter of this warp
     const int row = q4 * 32 + lane;           // query row = j * G + head in group
     const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
-    const int col = tid - 64;                 // 0..127: the column this thread zeroes
+    const uint32_t ocol = tmem + lane_off + kColO + (uint32_t)par * kD;
+    const uint32_t ocol_other = tmem + lane_off + kColO + (uint32_t)(par ^ 1) * kD;
+    const int col = (warp - 2 - 4 * par) * 32 + lane;   // column whose V row this thread zeroes
+    const float c2 = p.scale_log2;
     float m_used = -INFINITY, l = 0.f;
-    int t = 0;
-    while (!ctrl->abort_flag) {
+    int xcnt = 0;
+    bool pend_rel = false;
+    for (int t = par, own = 0; !ctrl->abort_flag; t += 2, ++own) {
       const int s = t % kStagesTC;
       if (!wait_or_abort(&ctrl->kv_full[s], (t / kStagesTC) & 1, ctrl, p.err)) break;
       const TileMeta m = ctrl->meta[s];
       if (m.unit < 0) break;
-      if (!wait_or_abort(&ctrl->s_full[t & 1], (t >> 1) & 1, ctrl, p.err)) break;
+      if (!wait_or_abort(&ctrl->s_full[par], own & 1, ctrl, p.err)) break;
       tc_fence_after();
-      if (m.first) {
+      const bool first_own = m.k < 2;
+      if (first_own) {
         m_used = -INFINITY;
         l = 0.f;
       }
       const int R = m.nq * p.G;
       const int j = row / p.G;
       const bool warp_active = q4 * 32 < R;
-      const int dcol = (m.ncp - m.tile * kPagesPerTile) * kPage;   // first draft column
-      const int dend = dcol + m.nd;
+      ColMask cm;
+      cm.dcol = (m.ncp - m.tile * kPagesPerTile) * kPage;   // first draft column
+      cm.dend = cm.dcol + m.nd;
+      cm.lim = m.lim0 + j - m.tile * kN;                     // cache columns <= lim visible
       bool resc = false;
       float fo = 1.f;
-      const uint32_t scol = tmem + lane_off + (uint32_t)(t & 1) * kN;
+      const uint32_t scol = tmem + lane_off + (uint32_t)par * kN;
       if (warp_active) {
-        float x[kN];
-        {
-          uint32_t r0[32], r1[32], r2[32], r3[32];
-          tmem_ld32(scol + 0, r0);
-          tmem_ld32(scol + 32, r1);
-          tmem_ld32(scol + 64, r2);
-          tmem_ld32(scol + 96, r3);
+        const bool masked = __any_sync(kFull, !(cm.dcol >= kN && cm.lim >= kN - 1));
+        // pass 1: row maximum of the raw scores over the visible columns
+        float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+        for (int c = 0; c < kN / 32; ++c) {
+          uint32_t r[32];
+          tmem_ld32(scol + c * 32, r);
           tmem_wait_ld();
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
-            x[i] = __uint_as_float(r0[i]);
-            x[32 + i] = __uint_as_float(r1[i]);
-            x[64 + i] = __uint_as_float(r2[i]);
-            x[96 + i] = __uint_as_float(r3[i]);
+            float v = __uint_as_float(r[i]);
+            if (masked && !cm.vis(c * 32 + i)) v = -INFINITY;
+            mx[i & 3] = fmaxf(mx[i & 3], v);
           }
         }
-        const int lim = m.lim0 + j - m.tile * kN;     // cache columns c <= lim are visible
-        float mt = -INFINITY;
-#pragma unroll
-        for (int c = 0; c < kN; ++c) {
-          const bool vis = (c < dcol) ? (c <= lim) : (c < dend);
-          x[c] = vis ? x[c] * p.scale_log2 : -INFINITY;
-          mt = fmaxf(mt, x[c]);
-        }
+        const float mt = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])) * c2;
         if (mt > m_used + kRescale) {
-          const float f = (m_used == -INFINITY) ? 0.f : exp2f(m_used - mt);
-          if (!m.first && m_used != -INFINITY) {
+          const float f = (m_used == -INFINITY) ? 0.f : ex2_approx(m_used - mt);
+          if (!first_own && m_used != -INFINITY) {
             resc = true;
             fo = f;
           }
           l *= f;
           m_used = mt;
         }
-        const float mu = (m_used == -INFINITY) ? 0.f : m_used;
-        float lsum = 0.f;
-        // P_hi of tokens [64h, 64h+64) -> packed columns [32h, 32h+32),
-        // P_lo -> [64 + 32h, 64 + 32h + 32); even token in the low half-word
+        const float mc = (m_used == -INFINITY) ? 0.f : m_used;
+        // pass 2: p = 2^(s*c - m), written back as P_hi / P_lo bf16 pairs:
+        // tokens [32c, 32c+32) -> packed columns [16c, 16c+16) (P_hi) and
+        // [64 + 16c, 64 + 16c + 16) (P_lo); even token in the low half-word
+        float ls[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-        for (int half = 0; half < 2; ++half) {
-          uint32_t wh[32], wl[32];
+        for (int c = 0; c < kN / 32; ++c) {
+          uint32_t r[32];
+          tmem_ld32(scol + 32 * c, r);
+          tmem_wait_ld();
+          uint32_t wh[16], wl[16];
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const float p0 = exp2f(x[64 * half + 2 * i] - mu);
-            const float p1 = exp2f(x[64 * half + 2 * i + 1] - mu);
-            lsum += p0 + p1;
+          for (int i = 0; i < 16; ++i) {
+            const int c0 = 32 * c + 2 * i;
+            float s0 = __uint_as_float(r[2 * i]);
+            float s1 = __uint_as_float(r[2 * i + 1]);
+            if (masked) {
+              if (!cm.vis(c0)) s0 = -INFINITY;
+              if (!cm.vis(c0 + 1)) s1 = -INFINITY;
+            }
+            const float p0 = ex2_approx(fmaf(s0, c2, -mc));
+            const float p1 = ex2_approx(fmaf(s1, c2, -mc));
+            ls[i & 3] += p0 + p1;
             const uint32_t h = pack_bf16x2(p0, p1);
             wh[i] = h;
             wl[i] = pack_bf16x2(p0 - bf16lo(h), p1 - bf16hi(h));
           }
-          tmem_st32(scol + 32 * half, wh);
-          tmem_st32(scol + 64 + 32 * half, wl);
+          tmem_st16(scol + 16 * c, wh);
+          tmem_st16(scol + 64 + 16 * c, wl);
         }
         tmem_wait_st();
-        l += lsum;
+        l += (ls[0] + ls[1]) + (ls[2] + ls[3]);
       }
       // V rows of columns nobody may see are zeroed, so that a probability of
       // 0 never meets a stale or NaN-poisoned row
       {
-        const bool valid = (col < dcol) ? (col < m.cvalid - m.tile * kN) : (col < dend);
+        const bool valid = (col < cm.dcol) ? (col < m.cvalid - m.tile * kN) : (col < cm.dend);
         if (!valid) {
           uint8_t* vb = smem + kOffStages + (size_t)s * kStageBytes + 2 * kHalf;
 #pragma unroll
@@ -536,133 +562,153 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
           fence_proxy_async_smem();
         }
       }
-      // the previous PV must be done before O is rescaled (and before the
-      // next one is issued on top of it)
-      if (t > 0 && !wait_or_abort(&ctrl->o_full, (t - 1) & 1, ctrl, p.err)) break;
+      // this group's previous PV must be done before its O is rescaled
+      if (own > 0 && !wait_or_abort(&ctrl->o_full[par], (own - 1) & 1, ctrl, p.err)) break;
+      // the first tile of a unit overwrites O: the other group's epilogue of
+      // the previous unit must have read it
+      if (first_own && pend_rel) {
+        if (!wait_or_abort(&ctrl->orel_bar[q4], (xcnt - 1) & 1, ctrl, p.err)) break;
+        pend_rel = false;
+      }
       tc_fence_after();
       if (warp_active && __any_sync(kFull, resc)) {
         const float f = resc ? fo : 1.f;
-        uint32_t r0[32], r1[32], r2[32], r3[32];
-        tmem_ld32(tmem + lane_off + kColO + 0, r0);
-        tmem_ld32(tmem + lane_off + kColO + 32, r1);
-        tmem_ld32(tmem + lane_off + kColO + 64, r2);
-        tmem_ld32(tmem + lane_off + kColO + 96, r3);
-        tmem_wait_ld();
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          r0[i] = __float_as_uint(__uint_as_float(r0[i]) * f);
-          r1[i] = __float_as_uint(__uint_as_float(r1[i]) * f);
-          r2[i] = __float_as_uint(__uint_as_float(r2[i]) * f);
-          r3[i] = __float_as_uint(__uint_as_float(r3[i]) * f);
+        for (int c = 0; c < kD / 32; ++c) {
+          uint32_t r[32];
+          tmem_ld32(ocol + c * 32, r);
+          tmem_wait_ld();
+#pragma unroll
+          for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * f);
+          tmem_st32(ocol + c * 32, r);
         }
-        tmem_st32(tmem + lane_off + kColO + 0, r0);
-        tmem_st32(tmem + lane_off + kColO + 32, r1);
-        tmem_st32(tmem + lane_off + kColO + 64, r2);
-        tmem_st32(tmem + lane_off + kColO + 96, r3);
         tmem_wait_st();
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&ctrl->p_full[t & 1]);
+      if (lane == 0) mbar_arrive(&ctrl->p_full[par]);
 
-      if (m.last) {
-        // ------------------------------------------------------ epilogue
-        if (!wait_or_abort(&ctrl->o_full, t & 1, ctrl, p.err)) break;
+      if (m.k + 2 >= m.ntu) {
+        // ------------------------------------------------ this group's last tile of the unit
+        if (!wait_or_abort(&ctrl->o_full[par], own & 1, ctrl, p.err)) break;
         tc_fence_after();
-        if (warp_active) {
-          const int REC = Rmax * (kD + 1);
-          const bool real = row < R;
-          const int qh = m.g * p.G + (row - j * p.G);
-          const size_t orow = ((size_t)m.b * p.W1 + j) * p.hq + qh;   // [b, j, head]
-          const float inv = (l > 0.f) ? 1.f / l : 0.f;
-          const float lse2 = (l > 0.f) ? m_used + log2f(l) : -INFINITY;
-          uint32_t r0[32], r1[32], r2[32], r3[32];
-          tmem_ld32(tmem + lane_off + kColO + 0, r0);
-          tmem_ld32(tmem + lane_off + kColO + 32, r1);
-          tmem_ld32(tmem + lane_off + kColO + 64, r2);
-          tmem_ld32(tmem + lane_off + kColO + 96, r3);
-          tmem_wait_ld();
-          if (m.nunits == 1) {
-            if (real) {
-              float* dst = p.out + orow * kD;
-#pragma unroll
-              for (int i = 0; i < 32; i += 4) {
-                *reinterpret_cast<float4*>(dst + i) =
-                    make_float4(__uint_as_float(r0[i]) * inv, __uint_as_float(r0[i + 1]) * inv,
-                                __uint_as_float(r0[i + 2]) * inv, __uint_as_float(r0[i + 3]) * inv);
-                *reinterpret_cast<float4*>(dst + 32 + i) =
-                    make_float4(__uint_as_float(r1[i]) * inv, __uint_as_float(r1[i + 1]) * inv,
-                                __uint_as_float(r1[i + 2]) * inv, __uint_as_float(r1[i + 3]) * inv);
-                *reinterpret_cast<float4*>(dst + 64 + i) =
-                    make_float4(__uint_as_float(r2[i]) * inv, __uint_as_float(r2[i + 1]) * inv,
-                                __uint_as_float(r2[i + 2]) * inv, __uint_as_float(r2[i + 3]) * inv);
-                *reinterpret_cast<float4*>(dst + 96 + i) =
-                    make_float4(__uint_as_float(r3[i]) * inv, __uint_as_float(r3[i + 1]) * inv,
-                                __uint_as_float(r3[i + 2]) * inv, __uint_as_float(r3[i + 3]) * inv);
-              }
-              if (p.lse != nullptr) p.lse[orow] = lse2 * kLn2;
-            }
-          } else {
-            // partial record, column-major [d][row] so that the rows of a warp
-            // store (and later load) contiguously
+        if (m.k != m.ntu - 1) {
+          // the other group owns the epilogue: hand over this row's statistics
+          ctrl->xm[q4][lane] = m_used;
+          ctrl->xl[q4][lane] = l;
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&ctrl->stats_bar[q4]);
+          pend_rel = true;
+          ++xcnt;
+        } else {
+          // ---------------------------------------------- epilogue (owner)
+          float mo = -INFINITY, lo = 0.f;
+          if (m.ntu >= 2) {
+            if (!wait_or_abort(&ctrl->stats_bar[q4], xcnt & 1, ctrl, p.err)) break;
+            tc_fence_after();
+            mo = ctrl->xm[q4][lane];
+            lo = ctrl->xl[q4][lane];
+          }
+          if (warp_active) {
+            const float M = fmaxf(m_used, lo > 0.f ? mo : -INFINITY);
+            const float fa = (l > 0.f) ? ex2_approx(m_used - M) : 0.f;
+            const float fb = (lo > 0.f) ? ex2_approx(mo - M) : 0.f;
+            const float Ls = l * fa + lo * fb;
+            const float inv = (Ls > 0.f) ? 1.f / Ls : 0.f;
+            const float lse2 = (Ls > 0.f) ? M + log2f(Ls) : -INFINITY;
+            const bool use_other = __any_sync(kFull, lo > 0.f);
+            const int REC = Rmax * (kD + 1);
+            const bool real = row < R;
+            const int qh = m.g * p.G + (row - j * p.G);
+            const size_t orow = ((size_t)m.b * p.W1 + j) * p.hq + qh;   // [b, j, head]
+            float* dst_out = p.out + orow * kD;
             float* rec = p.part + (size_t)(m.rec0 + m.chunk) * REC;
-            if (real) {
-#pragma unroll
-              for (int i = 0; i < 32; ++i) {
-                rec[(size_t)i * Rmax + row] = __uint_as_float(r0[i]) * inv;
-                rec[(size_t)(32 + i) * Rmax + row] = __uint_as_float(r1[i]) * inv;
-                rec[(size_t)(64 + i) * Rmax + row] = __uint_as_float(r2[i]) * inv;
-                rec[(size_t)(96 + i) * Rmax + row] = __uint_as_float(r3[i]) * inv;
-              }
-              rec[(size_t)kD * Rmax + row] = lse2;
-            }
-            __threadfence();
-            __syncwarp();
-            int last = 0;
-            if (lane == 0)
-              last = atomicAdd(&p.counters[(m.b * p.hkv + m.g) * 4 + q4], 1) == m.nunits - 1;
-            last = __shfl_sync(kFull, last, 0);
-            if (last) {
-              // this warp merges its rows over all units of the pair
-              __threadfence();
-              if (real) {
-                const float* base = p.part + (size_t)m.rec0 * REC;
-                float M = -INFINITY;
-                for (int c = 0; c < m.nunits; ++c)
-                  M = fmaxf(M, __ldcg(base + (size_t)c * REC + (size_t)kD * Rmax + row));
-                float S = 0.f;
-                for (int c = 0; c < m.nunits; ++c) {
-                  const float lc = __ldcg(base + (size_t)c * REC + (size_t)kD * Rmax + row);
-                  S += (lc == -INFINITY) ? 0.f : exp2f(lc - M);
-                }
-                const float invS = 1.f / S;
-                float* dst = p.out + orow * kD;
 #pragma unroll 1
-                for (int d0 = 0; d0 < kD; d0 += 32) {
-                  float acc[32];
+            for (int c = 0; c < kD / 16; ++c) {
+              uint32_t ra[16], rb[16];
+              tmem_ld16(ocol + c * 16, ra);
+              if (use_other) tmem_ld16(ocol_other + c * 16, rb);
+              tmem_wait_ld();
+              float v[16];
 #pragma unroll
-                  for (int i = 0; i < 32; ++i) acc[i] = 0.f;
-                  for (int c = 0; c < m.nunits; ++c) {
-                    const float* rc = base + (size_t)c * REC;
-                    const float lc = __ldcg(rc + (size_t)kD * Rmax + row);
-                    const float w = (lc == -INFINITY) ? 0.f : exp2f(lc - M) * invS;
-#pragma unroll
-                    for (int i = 0; i < 32; ++i)
-                      acc[i] = fmaf(w, __ldcg(rc + (size_t)(d0 + i) * Rmax + row), acc[i]);
-                  }
-#pragma unroll
-                  for (int i = 0; i < 32; i += 4)
-                    *reinterpret_cast<float4*>(dst + d0 + i) =
-                        make_float4(acc[i], acc[i + 1], acc[i + 2], acc[i + 3]);
-                }
-                if (p.lse != nullptr) p.lse[orow] = (M + log2f(S)) * kLn2;
+              for (int i = 0; i < 16; ++i) {
+                float x = __uint_as_float(ra[i]) * fa;
+                if (use_other && lo > 0.f) x = fmaf(__uint_as_float(rb[i]), fb, x);
+                v[i] = x * inv;
               }
-              if (lane == 0) p.counters[(m.b * p.hkv + m.g) * 4 + q4] = 0;
+              if (real) {
+                // final output row, or this unit's partial record (same
+                // row-major layout: [row][d] then the per-row log2-sum-exp)
+                float4* dp = reinterpret_cast<float4*>(
+                    (m.nunits == 1 ? dst_out : rec + (size_t)row * kD) + c * 16);
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                  dp[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+              }
             }
+            if (m.nunits == 1) {
+              if (real && p.lse != nullptr) p.lse[orow] = lse2 * kLn2;
+            } else {
+              if (real) rec[(size_t)kD * Rmax + row] = lse2;
+              __threadfence();
+              __syncwarp();
+              int lastw = 0;
+              if (lane == 0)
+                lastw = atomicAdd(&p.counters[(m.b * p.hkv + m.g) * 4 + q4], 1) == m.nunits - 1;
+              lastw = __shfl_sync(kFull, lastw, 0);
+              if (lastw) {
+                // this warp merges its rows over all units of the pair
+                __threadfence();
+                if (real) {
+                  const float* base = p.part + (size_t)m.rec0 * REC;
+                  float Mx = -INFINITY;
+                  for (int c = 0; c < m.nunits; ++c)
+                    Mx = fmaxf(Mx, __ldcg(base + (size_t)c * REC + (size_t)kD * Rmax + row));
+                  float S = 0.f;
+                  for (int c = 0; c < m.nunits; ++c) {
+                    const float lc = __ldcg(base + (size_t)c * REC + (size_t)kD * Rmax + row);
+                    S += (lc == -INFINITY) ? 0.f : ex2_approx(lc - Mx);
+                  }
+                  const float invS = 1.f / S;
+#pragma unroll 1
+                  for (int d0 = 0; d0 < kD; d0 += 16) {
+                    float acc[16];
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) acc[i] = 0.f;
+                    for (int c = 0; c < m.nunits; ++c) {
+                      const float* rc = base + (size_t)c * REC;
+                      const float lc = __ldcg(rc + (size_t)kD * Rmax + row);
+                      const float w = (lc == -INFINITY) ? 0.f : ex2_approx(lc - Mx) * invS;
+                      const float4* rp = reinterpret_cast<const float4*>(rc + (size_t)row * kD + d0);
+#pragma unroll
+                      for (int i = 0; i < 4; ++i) {
+                        const float4 x = __ldcg(rp + i);
+                        acc[4 * i] = fmaf(w, x.x, acc[4 * i]);
+                        acc[4 * i + 1] = fmaf(w, x.y, acc[4 * i + 1]);
+                        acc[4 * i + 2] = fmaf(w, x.z, acc[4 * i + 2]);
+                        acc[4 * i + 3] = fmaf(w, x.w, acc[4 * i + 3]);
+                      }
+                    }
+                    float4* dp = reinterpret_cast<float4*>(dst_out + d0);
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+                      dp[i] = make_float4(acc[4 * i], acc[4 * i + 1], acc[4 * i + 2], acc[4 * i + 3]);
+                  }
+                  if (p.lse != nullptr) p.lse[orow] = (Mx + log2f(S)) * kLn2;
+                }
+                if (lane == 0) p.counters[(m.b * p.hkv + m.g) * 4 + q4] = 0;
+              }
+            }
+          }
+          if (m.ntu >= 2) {
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&ctrl->orel_bar[q4]);
+            ++xcnt;
           }
         }
       }
-      ++t;
     }
   }
 
