@@ -432,15 +432,14 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
           const uint32_t pcol = tmem + (uint32_t)(tp & 1) * kN;
           const uint32_t ocol = tmem + kColO + (uint32_t)(tp & 1) * kD;
           const uint32_t vb = sbase + kOffStages + (uint32_t)sp * kStageBytes + 2 * kHalf;
+          // tokens [16kk, 16kk+16): P_hi at packed column 32*(kk/2) + 8*(kk%2),
+          // P_lo 16 columns further
 #pragma unroll
           for (int kk = 0; kk < kN / 16; ++kk) {
             const uint64_t b = smem_desc_sw128(vb + kk * 2048u, kHalf, 1024);
-            mma_ts(ocol, pcol + kk * 8, b, kIdescPV, !(prev_k < 2 && kk == 0));
-          }
-#pragma unroll
-          for (int kk = 0; kk < kN / 16; ++kk) {
-            const uint64_t b = smem_desc_sw128(vb + kk * 2048u, kHalf, 1024);
-            mma_ts(ocol, pcol + 64 + kk * 8, b, kIdescPV, 1);
+            const uint32_t a = pcol + 32 * (kk >> 1) + 8 * (kk & 1);
+            mma_ts(ocol, a, b, kIdescPV, !(prev_k < 2 && kk == 0));
+            mma_ts(ocol, a + 16, b, kIdescPV, 1);
           }
           mma_commit(&ctrl->o_full[tp & 1]);
           mma_commit(&ctrl->kv_empty[sp]);
@@ -517,8 +516,9 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
         }
         const float mc = (m_used == -INFINITY) ? 0.f : m_used;
         // pass 2: p = 2^(s*c - m), written back as P_hi / P_lo bf16 pairs:
-        // tokens [32c, 32c+32) -> packed columns [16c, 16c+16) (P_hi) and
-        // [64 + 16c, 64 + 16c + 16) (P_lo); even token in the low half-word
+        // tokens [32c, 32c+32) -> packed columns [32c, 32c+16) (P_hi) and
+        // [32c+16, 32c+32) (P_lo), i.e. inside the S columns this chunk has
+        // already consumed; even token in the low half-word
         float ls[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
         for (int c = 0; c < kN / 32; ++c) {
@@ -542,8 +542,8 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
             wh[i] = h;
             wl[i] = pack_bf16x2(p0 - bf16lo(h), p1 - bf16hi(h));
           }
-          tmem_st16(scol + 16 * c, wh);
-          tmem_st16(scol + 64 + 16 * c, wl);
+          tmem_st16(scol + 32 * c, wh);
+          tmem_st16(scol + 32 * c + 16, wl);
         }
         tmem_wait_st();
         l += (ls[0] + ls[1]) + (ls[2] + ls[3]);
