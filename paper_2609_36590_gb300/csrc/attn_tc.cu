@@ -248,8 +248,115 @@ struct ColMask {
   __device__ __forceinline__ bool vis(int c) const { return (c < dcol) ? (c <= lim) : (c < dend); }
 };
 
-__global__ void __launch_bounds__(kThreadsTC, 1)
-    attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
+// Epilogue of one unit for one warp's rows (run by the group that processed
+// the unit's last tile): combine the two groups' partial softmax states,
+// normalise, and write the output rows -- or this unit's partial record, in
+// which case the last warp (per pair and lane quarter) to finish merges all
+// records of the pair.  Kept out of line: it runs once per unit and needs
+// more registers than the per-tile loop.
+__device__ __noinline__ void unit_epilogue(const AttnTcParams& p, int b, int g, int nq, int rec0,
+                                           int chunk, int nunits, int row, int q4, int lane,
+                                           uint32_t ocol, uint32_t ocol_other, float m_used,
+                                           float l, float mo, float lo) {
+  const int Rmax = p.G * p.W1;
+  const int R = nq * p.G;
+  const int j = row / p.G;
+  const float M = fmaxf(m_used, lo > 0.f ? mo : -INFINITY);
+  const float fa = (l > 0.f) ? ex2_approx(m_used - M) : 0.f;
+  const float fb = (lo > 0.f) ? ex2_approx(mo - M) : 0.f;
+  const float Ls = l * fa + lo * fb;
+  const float inv = (Ls > 0.f) ? 1.f / Ls : 0.f;
+  const float lse2 = (Ls > 0.f) ? M + log2f(Ls) : -INFINITY;
+  const bool use_other = __any_sync(kFull, lo > 0.f);
+  const int REC = Rmax * (kD + 1);
+  const bool real = row < R;
+  const int qh = g * p.G + (row - j * p.G);
+  const size_t orow = ((size_t)b * p.W1 + j) * p.hq + qh;   // [b, j, head]
+  float* dst_out = p.out + orow * kD;
+  float* rec = p.part + (size_t)(rec0 + chunk) * REC;
+#pragma unroll 1
+  for (int c = 0; c < kD / 16; ++c) {
+    uint32_t ra[16], rb[16];
+    tmem_ld16(ocol + c * 16, ra);
+    if (use_other) tmem_ld16(ocol_other + c * 16, rb);
+    tmem_wait_ld();
+    float v[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      float x = __uint_as_float(ra[i]) * fa;
+      if (use_other && lo > 0.f) x = fmaf(__uint_as_float(rb[i]), fb, x);
+      v[i] = x * inv;
+    }
+    if (real) {
+      // final output row, or this unit's partial record (same
+      // row-major layout: [row][d] then the per-row log2-sum-exp)
+      float4* dp = reinterpret_cast<float4*>(
+          (nunits == 1 ? dst_out : rec + (size_t)row * kD) + c * 16);
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        dp[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+    }
+  }
+  if (nunits == 1) {
+    if (real && p.lse != nullptr) p.lse[orow] = lse2 * kLn2;
+  } else {
+    if (real) rec[(size_t)kD * Rmax + row] = lse2;
+    __threadfence();
+    __syncwarp();
+    int lastw = 0;
+    if (lane == 0)
+      lastw = atomicAdd(&p.counters[(b * p.hkv + g) * 4 + q4], 1) == nunits - 1;
+    lastw = __shfl_sync(kFull, lastw, 0);
+    if (lastw) {
+      // this warp merges its rows over all units of the pair
+      __threadfence();
+      if (real) {
+        const float* base = p.part + (size_t)rec0 * REC;
+        float Mx = -INFINITY;
+        for (int c = 0; c < nunits; ++c)
+          Mx = fmaxf(Mx, __ldcg(base + (size_t)c * REC + (size_t)kD * Rmax + row));
+        float S = 0.f;
+        for (int c = 0; c < nunits; ++c) {
+          const float lc = __ldcg(base + (size_t)c * REC + (size_t)kD * Rmax + row);
+          S += (lc == -INFINITY) ? 0.f : ex2_approx(lc - Mx);
+        }
+        const float invS = 1.f / S;
+#pragma unroll 1
+        for (int d0 = 0; d0 < kD; d0 += 16) {
+          float acc[16];
+#pragma unroll
+          for (int i = 0; i < 16; ++i) acc[i] = 0.f;
+          for (int c = 0; c < nunits; ++c) {
+            const float* rc = base + (size_t)c * REC;
+            const float lc = __ldcg(rc + (size_t)kD * Rmax + row);
+            const float w = (lc == -INFINITY) ? 0.f : ex2_approx(lc - Mx) * invS;
+            const float4* rp = reinterpret_cast<const float4*>(rc + (size_t)row * kD + d0);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              const float4 x = __ldcg(rp + i);
+              acc[4 * i] = fmaf(w, x.x, acc[4 * i]);
+              acc[4 * i + 1] = fmaf(w, x.y, acc[4 * i + 1]);
+              acc[4 * i + 2] = fmaf(w, x.z, acc[4 * i + 2]);
+              acc[4 * i + 3] = fmaf(w, x.w, acc[4 * i + 3]);
+            }
+          }
+          float4* dp = reinterpret_cast<float4*>(dst_out + d0);
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+            dp[i] = make_float4(acc[4 * i], acc[4 * i + 1], acc[4 * i + 2], acc[4 * i + 3]);
+        }
+        if (p.lse != nullptr) p.lse[orow] = (Mx + log2f(S)) * kLn2;
+      }
+      if (lane == 0) p.counters[(b * p.hkv + g) * 4 + q4] = 0;
+    }
+  }
+}
+
+// No __launch_bounds__: with it ptxas budgets the 320-thread block like a
+// 384-thread one and spills in the per-tile loop; without it the kernel fits
+// in 168 registers with no spills (a launch that did not fit would fail with
+// an error, never run).
+__global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
                    const __grid_constant__ CUtensorMap tm_k,
                    const __grid_constant__ CUtensorMap tm_v,
                    const __grid_constant__ CUtensorMap tm_dk,
@@ -610,97 +717,9 @@ __global__ void __launch_bounds__(kThreadsTC, 1)
             mo = ctrl->xm[q4][lane];
             lo = ctrl->xl[q4][lane];
           }
-          if (warp_active) {
-            const float M = fmaxf(m_used, lo > 0.f ? mo : -INFINITY);
-            const float fa = (l > 0.f) ? ex2_approx(m_used - M) : 0.f;
-            const float fb = (lo > 0.f) ? ex2_approx(mo - M) : 0.f;
-            const float Ls = l * fa + lo * fb;
-            const float inv = (Ls > 0.f) ? 1.f / Ls : 0.f;
-            const float lse2 = (Ls > 0.f) ? M + log2f(Ls) : -INFINITY;
-            const bool use_other = __any_sync(kFull, lo > 0.f);
-            const int REC = Rmax * (kD + 1);
-            const bool real = row < R;
-            const int qh = m.g * p.G + (row - j * p.G);
-            const size_t orow = ((size_t)m.b * p.W1 + j) * p.hq + qh;   // [b, j, head]
-            float* dst_out = p.out + orow * kD;
-            float* rec = p.part + (size_t)(m.rec0 + m.chunk) * REC;
-#pragma unroll 1
-            for (int c = 0; c < kD / 16; ++c) {
-              uint32_t ra[16], rb[16];
-              tmem_ld16(ocol + c * 16, ra);
-              if (use_other) tmem_ld16(ocol_other + c * 16, rb);
-              tmem_wait_ld();
-              float v[16];
-#pragma unroll
-              for (int i = 0; i < 16; ++i) {
-                float x = __uint_as_float(ra[i]) * fa;
-                if (use_other && lo > 0.f) x = fmaf(__uint_as_float(rb[i]), fb, x);
-                v[i] = x * inv;
-              }
-              if (real) {
-                // final output row, or this unit's partial record (same
-                // row-major layout: [row][d] then the per-row log2-sum-exp)
-                float4* dp = reinterpret_cast<float4*>(
-                    (m.nunits == 1 ? dst_out : rec + (size_t)row * kD) + c * 16);
-#pragma unroll
-                for (int i = 0; i < 4; ++i)
-                  dp[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
-              }
-            }
-            if (m.nunits == 1) {
-              if (real && p.lse != nullptr) p.lse[orow] = lse2 * kLn2;
-            } else {
-              if (real) rec[(size_t)kD * Rmax + row] = lse2;
-              __threadfence();
-              __syncwarp();
-              int lastw = 0;
-              if (lane == 0)
-                lastw = atomicAdd(&p.counters[(m.b * p.hkv + m.g) * 4 + q4], 1) == m.nunits - 1;
-              lastw = __shfl_sync(kFull, lastw, 0);
-              if (lastw) {
-                // this warp merges its rows over all units of the pair
-                __threadfence();
-                if (real) {
-                  const float* base = p.part + (size_t)m.rec0 * REC;
-                  float Mx = -INFINITY;
-                  for (int c = 0; c < m.nunits; ++c)
-                    Mx = fmaxf(Mx, __ldcg(base + (size_t)c * REC + (size_t)kD * Rmax + row));
-                  float S = 0.f;
-                  for (int c = 0; c < m.nunits; ++c) {
-                    const float lc = __ldcg(base + (size_t)c * REC + (size_t)kD * Rmax + row);
-                    S += (lc == -INFINITY) ? 0.f : ex2_approx(lc - Mx);
-                  }
-                  const float invS = 1.f / S;
-#pragma unroll 1
-                  for (int d0 = 0; d0 < kD; d0 += 16) {
-                    float acc[16];
-#pragma unroll
-                    for (int i = 0; i < 16; ++i) acc[i] = 0.f;
-                    for (int c = 0; c < m.nunits; ++c) {
-                      const float* rc = base + (size_t)c * REC;
-                      const float lc = __ldcg(rc + (size_t)kD * Rmax + row);
-                      const float w = (lc == -INFINITY) ? 0.f : ex2_approx(lc - Mx) * invS;
-                      const float4* rp = reinterpret_cast<const float4*>(rc + (size_t)row * kD + d0);
-#pragma unroll
-                      for (int i = 0; i < 4; ++i) {
-                        const float4 x = __ldcg(rp + i);
-                        acc[4 * i] = fmaf(w, x.x, acc[4 * i]);
-                        acc[4 * i + 1] = fmaf(w, x.y, acc[4 * i + 1]);
-                        acc[4 * i + 2] = fmaf(w, x.z, acc[4 * i + 2]);
-                        acc[4 * i + 3] = fmaf(w, x.w, acc[4 * i + 3]);
-                      }
-                    }
-                    float4* dp = reinterpret_cast<float4*>(dst_out + d0);
-#pragma unroll
-                    for (int i = 0; i < 4; ++i)
-                      dp[i] = make_float4(acc[4 * i], acc[4 * i + 1], acc[4 * i + 2], acc[4 * i + 3]);
-                  }
-                  if (p.lse != nullptr) p.lse[orow] = (Mx + log2f(S)) * kLn2;
-                }
-                if (lane == 0) p.counters[(m.b * p.hkv + m.g) * 4 + q4] = 0;
-              }
-            }
-          }
+          if (warp_active)
+            unit_epilogue(p, m.b, m.g, m.nq, m.rec0, m.chunk, m.nunits, row, q4, lane, ocol,
+                          ocol_other, m_used, l, mo, lo);
           if (m.ntu >= 2) {
             tc_fence_before();
             __syncwarp();
