@@ -599,7 +599,9 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
         const bool masked = __any_sync(kFull, !(cm.dcol >= kN && cm.lim >= kN - 1));
         // pass 1: row maximum of the raw scores over the visible columns
         float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-#pragma unroll
+        // chunk loops stay rolled: the fully unrolled softmax overflowed the
+        // instruction cache and stalled on instruction fetch
+#pragma unroll 1
         for (int c = 0; c < kN / 32; ++c) {
           uint32_t r[32];
           tmem_ld32(scol + c * 32, r);
@@ -627,7 +629,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
         // [32c+16, 32c+32) (P_lo), i.e. inside the S columns this chunk has
         // already consumed; even token in the low half-word
         float ls[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
+#pragma unroll 1
         for (int c = 0; c < kN / 32; ++c) {
           uint32_t r[32];
           tmem_ld32(scol + 32 * c, r);
@@ -680,7 +682,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
       tc_fence_after();
       if (warp_active && __any_sync(kFull, resc)) {
         const float f = resc ? fo : 1.f;
-#pragma unroll
+#pragma unroll 1
         for (int c = 0; c < kD / 32; ++c) {
           uint32_t r[32];
           tmem_ld32(ocol + c * 32, r);
