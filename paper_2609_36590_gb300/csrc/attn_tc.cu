@@ -102,12 +102,13 @@ struct Ctrl {
 constexpr size_t kSmemTC = kOffCtrl + sizeof(Ctrl) + 1024;   // + alignment slack
 static_assert(kSmemTC <= 232448, "shared memory budget");
 
+// Bounded wait (about 2 s) on an mbarrier phase; the waiting thread sleeps in
+// hardware between tries.  Gives up early if another role has aborted.
 __device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, Ctrl* c,
                                               int32_t* err) {
-  for (uint32_t i = 0; i < kSpinLimit; ++i) {
-    if (mbar_try_wait(bar, parity)) return true;
+  for (uint32_t i = 0; i < kSuspendTries; ++i) {
+    if (mbar_try_wait_sleep(bar, parity, kSuspendNs)) return true;
     if (c->abort_flag) return false;
-    if (i >= 32) __nanosleep(64);
   }
   c->abort_flag = 1;
   raise_err(err, SEED_DEVERR_TIMEOUT);

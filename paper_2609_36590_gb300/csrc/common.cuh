@@ -11,6 +11,8 @@ namespace seedk {
 
 constexpr int kPage = 16;                 // tokens per KV page (page_size)
 constexpr uint32_t kSpinLimit = 1u << 22; // polls before a wait gives up
+constexpr uint32_t kSuspendNs = 500000;   // per-try sleep bound of a suspending wait
+constexpr uint32_t kSuspendTries = 4000;  // suspending tries before a wait gives up (~2 s)
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -48,6 +50,21 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
       "selp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(ok)
       : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Like mbar_try_wait, but the thread sleeps in hardware (up to `ns`
+// nanoseconds) until the phase completes instead of returning at once, so
+// waiting warps stop issuing instructions.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t* bar, uint32_t parity, uint32_t ns) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity), "r"(ns)
       : "memory");
   return ok != 0;
 }
