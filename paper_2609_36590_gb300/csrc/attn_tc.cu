@@ -103,9 +103,11 @@ constexpr size_t kSmemTC = kOffCtrl + sizeof(Ctrl) + 1024;   // + alignment slac
 static_assert(kSmemTC <= 232448, "shared memory budget");
 
 // Bounded wait (about 2 s) on an mbarrier phase; the waiting thread sleeps in
-// hardware between tries.  Gives up early if another role has aborted.
-__device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, Ctrl* c,
-                                              int32_t* err) {
+// hardware between tries.  Gives up early if another role has aborted.  Out of
+// line, like the other cold helpers below: the kernel's code must stay small
+// enough for the instruction cache, or its warps stall on instruction fetch.
+__device__ __noinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, Ctrl* c,
+                                           int32_t* err) {
   for (uint32_t i = 0; i < kSuspendTries; ++i) {
     if (mbar_try_wait_sleep(bar, parity, kSuspendNs)) return true;
     if (c->abort_flag) return false;
@@ -152,7 +154,7 @@ struct Plan {
   int tpu, full_total, units;
 };
 
-__device__ Plan make_plan(const AttnTcParams& p, int lane) {
+__device__ __noinline__ Plan make_plan(const AttnTcParams& p, int lane) {
   long long tot = 0;
   for (int b = lane; b < p.B; b += 32) tot += seq_of(p, b).tiles;
   for (int o = 16; o; o >>= 1) tot += __shfl_xor_sync(kFull, tot, o);
@@ -182,7 +184,8 @@ struct UnitInfo {
 // Warp-cooperative: map dense unit index u to (b, g, chunk).  Units
 // [0, full_total) are the full-size units (tpu tiles) of all pairs, the rest
 // the ragged last units.  Record indices follow (b, g, chunk) order.
-__device__ UnitInfo lookup_unit(const AttnTcParams& p, const Plan& pl, int u, int lane) {
+__device__ __noinline__ UnitInfo lookup_unit(const AttnTcParams& p, const Plan& pl, int u,
+                                             int lane) {
   const bool full_phase = u < pl.full_total;
   const int target = full_phase ? u : u - pl.full_total;
   int base1 = 0, base2 = 0;
