@@ -35,8 +35,10 @@
 // the last warp to finish merges them in unit order, so results are
 // deterministic.
 //
-// Warp roles (192 threads): warp 0 TMA producer and scheduler, warp 1 MMA
-// issuer and TMEM owner, warps 2-5 softmax / epilogue.  Every wait is bounded;
+// Warp roles (384 threads): warps 0-7 softmax / epilogue (two groups of four,
+// one warp per TMEM lane quarter), warp 10 TMA producer and scheduler, warp 11
+// MMA issuer and TMEM owner; warps 8-9 only keep the role warps off the
+// sub-partition of lane quarter 0.  Every wait is bounded;
 // a wait that gives up raises SEED_DEVERR_TIMEOUT and all roles drain out.
 #include <cuda.h>
 #include <cuda_runtime.h>
@@ -56,7 +58,8 @@ constexpr int kD = 128;
 constexpr int kN = 128;                      // tokens (columns) per tile
 constexpr int kPagesPerTile = kN / kPage;    // 8
 constexpr int kStagesTC = 3;
-constexpr int kThreadsTC = 320;   // producer, MMA, 2 x 4 softmax warps
+constexpr int kThreadsTC = 384;   // warps 0-7 softmax, 8-9 idle, 10 TMA producer, 11 MMA
+constexpr int kWarpProducer = 10, kWarpMma = 11;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kColO = 256;              // O accumulators: [256, 384) and [384, 512)
 constexpr float kRescale = 8.0f;
@@ -391,7 +394,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
     ctrl->abort_flag = 0;
     fence_mbar_init();
   }
-  if (warp == 1) {
+  if (warp == kWarpMma) {
     tmem_alloc(&ctrl->tmem_base, kTmemCols);
     tmem_relinquish();
   }
@@ -401,7 +404,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
   const uint32_t tmem = ctrl->tmem_base;
   const int Rmax = p.G * p.W1;
 
-  if (warp == 0) {
+  if (warp == kWarpProducer) {
     // ---------------------------------------------------------- producer
     if (lane == 0) {
       tma_prefetch_desc(&tm_q);
@@ -475,20 +478,18 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
             if (pids[pp] >= 0 || pp == dslot) bytes += 4u * 2048u;
           mbar_arrive_expect_tx(&ctrl->kv_full[s], bytes);
           uint8_t* st = smem + kOffStages + (size_t)s * kStageBytes;
-#pragma unroll
+#pragma unroll 1
           for (int pp = 0; pp < kPagesPerTile; ++pp) {
+            const bool is_draft = pids[pp] < 0 && pp == dslot;
+            if (pids[pp] < 0 && !is_draft) continue;
+            const CUtensorMap* mk = is_draft ? &tm_dk : &tm_k;
+            const CUtensorMap* mv = is_draft ? &tm_dv : &tm_v;
+            const int w = is_draft ? ui.b : pids[pp];
             const uint32_t off = pp * 2048u;
-            if (pids[pp] >= 0) {
-              tma_load_4d(st + 0 * kHalf + off, &tm_k, 0, 0, ui.g, pids[pp], &ctrl->kv_full[s]);
-              tma_load_4d(st + 1 * kHalf + off, &tm_k, 64, 0, ui.g, pids[pp], &ctrl->kv_full[s]);
-              tma_load_4d(st + 2 * kHalf + off, &tm_v, 0, 0, ui.g, pids[pp], &ctrl->kv_full[s]);
-              tma_load_4d(st + 3 * kHalf + off, &tm_v, 64, 0, ui.g, pids[pp], &ctrl->kv_full[s]);
-            } else if (pp == dslot) {
-              tma_load_4d(st + 0 * kHalf + off, &tm_dk, 0, 0, ui.g, ui.b, &ctrl->kv_full[s]);
-              tma_load_4d(st + 1 * kHalf + off, &tm_dk, 64, 0, ui.g, ui.b, &ctrl->kv_full[s]);
-              tma_load_4d(st + 2 * kHalf + off, &tm_dv, 0, 0, ui.g, ui.b, &ctrl->kv_full[s]);
-              tma_load_4d(st + 3 * kHalf + off, &tm_dv, 64, 0, ui.g, ui.b, &ctrl->kv_full[s]);
-            }
+            tma_load_4d(st + 0 * kHalf + off, mk, 0, 0, ui.g, w, &ctrl->kv_full[s]);
+            tma_load_4d(st + 1 * kHalf + off, mk, 64, 0, ui.g, w, &ctrl->kv_full[s]);
+            tma_load_4d(st + 2 * kHalf + off, mv, 0, 0, ui.g, w, &ctrl->kv_full[s]);
+            tma_load_4d(st + 3 * kHalf + off, mv, 64, 0, ui.g, w, &ctrl->kv_full[s]);
           }
         }
         __syncwarp();
@@ -504,7 +505,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
         mbar_arrive(&ctrl->kv_full[s]);
       }
     }
-  } else if (warp == 1) {
+  } else if (warp == kWarpMma) {
     // ---------------------------------------------------------- MMA issuer
     if (lane == 0) {
       int t = 0, uo = 0, prev_k = 0;
@@ -525,7 +526,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
           tc_fence_after();
           const uint32_t d = tmem + (uint32_t)(t & 1) * kN;
           const uint32_t kb = sbase + kOffStages + (uint32_t)s * kStageBytes;
-#pragma unroll
+#pragma unroll 1
           for (int kk = 0; kk < kD / 16; ++kk) {
             const uint32_t h = kk >> 2, off = (kk & 3) * 32;
             const uint64_t a = smem_desc_sw128(sbase + h * kHalf + off, 16, 1024);
@@ -545,7 +546,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
           const uint32_t vb = sbase + kOffStages + (uint32_t)sp * kStageBytes + 2 * kHalf;
           // tokens [16kk, 16kk+16): P_hi at packed column 32*(kk/2) + 8*(kk%2),
           // P_lo 16 columns further
-#pragma unroll
+#pragma unroll 1
           for (int kk = 0; kk < kN / 16; ++kk) {
             const uint64_t b = smem_desc_sw128(vb + kk * 2048u, kHalf, 1024);
             const uint32_t a = pcol + 32 * (kk >> 1) + 8 * (kk & 1);
@@ -562,17 +563,19 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
       }
     }
     __syncwarp();
-  } else {
+  } else if (warp < 8) {
     // ---------------------------------------------------------- softmax
-    // Warps 2-5 take the even tiles of the CTA, warps 6-9 the odd ones; each
-    // group keeps its own running max, sum and O accumulator per row.
-    const int par = (warp - 2) >> 2;
+    // Warps 0-3 take the even tiles of the CTA, warps 4-7 the odd ones; each
+    // group keeps its own running max, sum and O accumulator per row.  (The
+    // producer and MMA warps sit on the SM sub-partitions of lane quarters 2
+    // and 3, away from quarter 0, which holds the rows of small tiles.)
+    const int par = warp >> 2;
     const int q4 = warp & 3;                  // TMEM lane quarter of this warp
     const int row = q4 * 32 + lane;           // query row = j * G + head in group
     const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
     const uint32_t ocol = tmem + lane_off + kColO + (uint32_t)par * kD;
     const uint32_t ocol_other = tmem + lane_off + kColO + (uint32_t)(par ^ 1) * kD;
-    const int col = (warp - 2 - 4 * par) * 32 + lane;   // column whose V row this thread zeroes
+    const int col = (warp - 4 * par) * 32 + lane;   // column whose V row this thread zeroes
     const float c2 = p.scale_log2;
     float m_used = -INFINITY, l = 0.f;
     int xcnt = 0;
@@ -667,7 +670,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
         const bool valid = (col < cm.dcol) ? (col < m.cvalid - m.tile * kN) : (col < cm.dend);
         if (!valid) {
           uint8_t* vb = smem + kOffStages + (size_t)s * kStageBytes + 2 * kHalf;
-#pragma unroll
+#pragma unroll 1
           for (int ch = 0; ch < 8; ++ch) {
             *reinterpret_cast<uint4*>(vb + col * 128 + ch * 16) = make_uint4(0, 0, 0, 0);
             *reinterpret_cast<uint4*>(vb + kHalf + col * 128 + ch * 16) = make_uint4(0, 0, 0, 0);
@@ -740,7 +743,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
   // ------------------------------------------------------------ teardown
   tc_fence_before();
   __syncthreads();
-  if (warp == 1) {
+  if (warp == kWarpMma) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }
