@@ -249,11 +249,79 @@ __device__ __noinline__ UnitInfo lookup_unit(const AttnTcParams& p, const Plan& 
 }
 
 // ------------------------------------------------------------- the kernel
-// One softmax row: the visible-column mask of tile `m` for query j.
+// One softmax row: the visible columns of a tile for query j are the cache
+// columns c <= lim (c < dcol) and the draft columns dcol <= c < dend.
 struct ColMask {
   int dcol, dend, lim;
   __device__ __forceinline__ bool vis(int c) const { return (c < dcol) ? (c <= lim) : (c < dend); }
+  // bit i set <=> column c0 + i is visible
+  __device__ __forceinline__ uint32_t bits(int c0) const {
+    const int nc = min(max(min(lim, dcol - 1) - c0 + 1, 0), 32);
+    const int lo = min(max(dcol - c0, 0), 32), hi = min(max(dend - c0, 0), 32);
+    const uint32_t mc = nc == 32 ? 0xffffffffu : ((1u << nc) - 1u);
+    const uint32_t mh = hi == 32 ? 0xffffffffu : ((1u << hi) - 1u);
+    const uint32_t ml = lo == 32 ? 0xffffffffu : ((1u << lo) - 1u);
+    return mc | (mh & ~ml);
+  }
 };
+
+// Pass 1 of a tile's softmax row: maximum of the raw scores over the visible
+// columns.  MASKED = false for the (common) tiles every column of which is
+// visible, so that their loop carries no per-column test.
+template <bool MASKED>
+__device__ __forceinline__ float row_max(uint32_t scol, const ColMask& cm) {
+  float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll 1
+  for (int c = 0; c < kN / 32; ++c) {
+    uint32_t r[32];
+    tmem_ld32(scol + c * 32, r);
+    tmem_wait_ld();
+    const uint32_t bits = MASKED ? cm.bits(32 * c) : 0xffffffffu;
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      float v = __uint_as_float(r[i]);
+      if (MASKED) v = ((bits >> i) & 1u) ? v : -INFINITY;
+      mx[i & 3] = fmaxf(mx[i & 3], v);
+    }
+  }
+  return fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+}
+
+// Pass 2: p = 2^(s*c2 - mc) written back as P_hi / P_lo bf16 pairs -- tokens
+// [32c, 32c+32) to packed columns [32c, 32c+16) (P_hi) and [32c+16, 32c+32)
+// (P_lo), i.e. inside the S columns this chunk has already consumed; even
+// token in the low half-word.  Returns the sum of the p.
+template <bool MASKED>
+__device__ __forceinline__ float row_p(uint32_t scol, const ColMask& cm, float c2, float mc) {
+  float ls[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 1
+  for (int c = 0; c < kN / 32; ++c) {
+    uint32_t r[32];
+    tmem_ld32(scol + 32 * c, r);
+    tmem_wait_ld();
+    const uint32_t bits = MASKED ? cm.bits(32 * c) : 0xffffffffu;
+    uint32_t wh[16], wl[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      float s0 = __uint_as_float(r[2 * i]);
+      float s1 = __uint_as_float(r[2 * i + 1]);
+      if (MASKED) {
+        s0 = ((bits >> (2 * i)) & 1u) ? s0 : -INFINITY;
+        s1 = ((bits >> (2 * i + 1)) & 1u) ? s1 : -INFINITY;
+      }
+      const float p0 = ex2_approx(fmaf(s0, c2, -mc));
+      const float p1 = ex2_approx(fmaf(s1, c2, -mc));
+      ls[i & 3] += p0 + p1;
+      const uint32_t h = pack_bf16x2(p0, p1);
+      wh[i] = h;
+      wl[i] = pack_bf16x2(p0 - bf16lo(h), p1 - bf16hi(h));
+    }
+    tmem_st16(scol + 32 * c, wh);
+    tmem_st16(scol + 32 * c + 16, wl);
+  }
+  tmem_wait_st();
+  return (ls[0] + ls[1]) + (ls[2] + ls[3]);
+}
 
 // Epilogue of one unit for one warp's rows (run by the group that processed
 // the unit's last tile): combine the two groups' partial softmax states,
@@ -319,6 +387,8 @@ __device__ __noinline__ void unit_epilogue(const AttnTcParams& p, int b, int g, 
       __threadfence();
       if (real) {
         const float* base = p.part + (size_t)rec0 * REC;
+        // log2-sum-exps of all units first (independent loads), then the rows
+        // in 32-column slices with up to 4 units' loads in flight at a time
         float Mx = -INFINITY;
         for (int c = 0; c < nunits; ++c)
           Mx = fmaxf(Mx, __ldcg(base + (size_t)c * REC + (size_t)kD * Rmax + row));
@@ -329,28 +399,37 @@ __device__ __noinline__ void unit_epilogue(const AttnTcParams& p, int b, int g, 
         }
         const float invS = 1.f / S;
 #pragma unroll 1
-        for (int d0 = 0; d0 < kD; d0 += 16) {
-          float acc[16];
+        for (int d0 = 0; d0 < kD; d0 += 32) {
+          float4 acc[8];
 #pragma unroll
-          for (int i = 0; i < 16; ++i) acc[i] = 0.f;
-          for (int c = 0; c < nunits; ++c) {
-            const float* rc = base + (size_t)c * REC;
-            const float lc = __ldcg(rc + (size_t)kD * Rmax + row);
-            const float w = (lc == -INFINITY) ? 0.f : ex2_approx(lc - Mx) * invS;
-            const float4* rp = reinterpret_cast<const float4*>(rc + (size_t)row * kD + d0);
+          for (int i = 0; i < 8; ++i) acc[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 1
+          for (int c0 = 0; c0 < nunits; c0 += 4) {
+            float4 x[4][8];
+            float w[4];
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              const float4 x = __ldcg(rp + i);
-              acc[4 * i] = fmaf(w, x.x, acc[4 * i]);
-              acc[4 * i + 1] = fmaf(w, x.y, acc[4 * i + 1]);
-              acc[4 * i + 2] = fmaf(w, x.z, acc[4 * i + 2]);
-              acc[4 * i + 3] = fmaf(w, x.w, acc[4 * i + 3]);
+            for (int u = 0; u < 4; ++u) {
+              const int c = c0 + u;
+              const float* rc = base + (size_t)min(c, nunits - 1) * REC;
+              const float lc = __ldcg(rc + (size_t)kD * Rmax + row);
+              w[u] = (c >= nunits || lc == -INFINITY) ? 0.f : ex2_approx(lc - Mx) * invS;
+              const float4* rp = reinterpret_cast<const float4*>(rc + (size_t)row * kD + d0);
+#pragma unroll
+              for (int i = 0; i < 8; ++i) x[u][i] = __ldcg(rp + i);
             }
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+#pragma unroll
+              for (int i = 0; i < 8; ++i) {
+                acc[i].x = fmaf(w[u], x[u][i].x, acc[i].x);
+                acc[i].y = fmaf(w[u], x[u][i].y, acc[i].y);
+                acc[i].z = fmaf(w[u], x[u][i].z, acc[i].z);
+                acc[i].w = fmaf(w[u], x[u][i].w, acc[i].w);
+              }
           }
           float4* dp = reinterpret_cast<float4*>(dst_out + d0);
 #pragma unroll
-          for (int i = 0; i < 4; ++i)
-            dp[i] = make_float4(acc[4 * i], acc[4 * i + 1], acc[4 * i + 2], acc[4 * i + 3]);
+          for (int i = 0; i < 8; ++i) dp[i] = acc[i];
         }
         if (p.lse != nullptr) p.lse[orow] = (Mx + log2f(S)) * kLn2;
       }
@@ -604,23 +683,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
       const uint32_t scol = tmem + lane_off + (uint32_t)par * kN;
       if (warp_active) {
         const bool masked = __any_sync(kFull, !(cm.dcol >= kN && cm.lim >= kN - 1));
-        // pass 1: row maximum of the raw scores over the visible columns
-        float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-        // chunk loops stay rolled: the fully unrolled softmax overflowed the
-        // instruction cache and stalled on instruction fetch
-#pragma unroll 1
-        for (int c = 0; c < kN / 32; ++c) {
-          uint32_t r[32];
-          tmem_ld32(scol + c * 32, r);
-          tmem_wait_ld();
-#pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            float v = __uint_as_float(r[i]);
-            if (masked && !cm.vis(c * 32 + i)) v = -INFINITY;
-            mx[i & 3] = fmaxf(mx[i & 3], v);
-          }
-        }
-        const float mt = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])) * c2;
+        const float mt = (masked ? row_max<true>(scol, cm) : row_max<false>(scol, cm)) * c2;
         if (mt > m_used + kRescale) {
           const float f = (m_used == -INFINITY) ? 0.f : ex2_approx(m_used - mt);
           if (!first_own && m_used != -INFINITY) {
@@ -631,38 +694,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
           m_used = mt;
         }
         const float mc = (m_used == -INFINITY) ? 0.f : m_used;
-        // pass 2: p = 2^(s*c - m), written back as P_hi / P_lo bf16 pairs:
-        // tokens [32c, 32c+32) -> packed columns [32c, 32c+16) (P_hi) and
-        // [32c+16, 32c+32) (P_lo), i.e. inside the S columns this chunk has
-        // already consumed; even token in the low half-word
-        float ls[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll 1
-        for (int c = 0; c < kN / 32; ++c) {
-          uint32_t r[32];
-          tmem_ld32(scol + 32 * c, r);
-          tmem_wait_ld();
-          uint32_t wh[16], wl[16];
-#pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            const int c0 = 32 * c + 2 * i;
-            float s0 = __uint_as_float(r[2 * i]);
-            float s1 = __uint_as_float(r[2 * i + 1]);
-            if (masked) {
-              if (!cm.vis(c0)) s0 = -INFINITY;
-              if (!cm.vis(c0 + 1)) s1 = -INFINITY;
-            }
-            const float p0 = ex2_approx(fmaf(s0, c2, -mc));
-            const float p1 = ex2_approx(fmaf(s1, c2, -mc));
-            ls[i & 3] += p0 + p1;
-            const uint32_t h = pack_bf16x2(p0, p1);
-            wh[i] = h;
-            wl[i] = pack_bf16x2(p0 - bf16lo(h), p1 - bf16hi(h));
-          }
-          tmem_st16(scol + 32 * c, wh);
-          tmem_st16(scol + 32 * c + 16, wl);
-        }
-        tmem_wait_st();
-        l += (ls[0] + ls[1]) + (ls[2] + ls[3]);
+        l += masked ? row_p<true>(scol, cm, c2, mc) : row_p<false>(scol, cm, c2, mc);
       }
       // V rows of columns nobody may see are zeroed, so that a probability of
       // 0 never meets a stale or NaN-poisoned row
