@@ -586,59 +586,77 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
     }
   } else if (warp == kWarpMma) {
     // ---------------------------------------------------------- MMA issuer
+    // An event loop over two streams: S(ts) = Q K^T of the next loaded tile
+    // and PV(tp) of the next tile whose probabilities are written.  Either is
+    // issued as soon as it is ready; the only orderings kept are PV(t) after
+    // S(t) and S(t) after PV(t-2) (S(t) overwrites P(t-2) in the same TMEM
+    // columns; one thread's MMAs execute in issue order).
     if (lane == 0) {
-      int t = 0, uo = 0, prev_k = 0;
-      bool have_prev = false;
-      while (true) {
-        const int s = t % kStagesTC;
-        if (!wait_or_abort(&ctrl->kv_full[s], (t / kStagesTC) & 1, ctrl, p.err)) break;
-        const int unit = ctrl->meta[s].unit;
-        const int k = ctrl->meta[s].k;
-        const int last = ctrl->meta[s].k == ctrl->meta[s].ntu - 1;
-        if (unit >= 0) {
-          if (k == 0) {
-            if (!wait_or_abort(&ctrl->q_full, uo & 1, ctrl, p.err)) break;
-            ++uo;
-          }
-          // S buffer t&1 is free once PV(t-2) has consumed its probabilities
-          if (t >= 2 && !wait_or_abort(&ctrl->o_full[t & 1], ((t - 2) >> 1) & 1, ctrl, p.err)) break;
-          tc_fence_after();
-          const uint32_t d = tmem + (uint32_t)(t & 1) * kN;
-          const uint32_t kb = sbase + kOffStages + (uint32_t)s * kStageBytes;
+      int ts = 0, tp = 0, uo = 0, t_end = 1 << 30;
+      int k_of[kStagesTC];               // tile index within its unit, per stage
+      uint32_t idle = 0;
+      while (tp < t_end && !ctrl->abort_flag) {
+        bool did = false;
+        if (ts < t_end && ts <= tp + 1) {
+          const int s = ts % kStagesTC;
+          if (mbar_test(&ctrl->kv_full[s], (ts / kStagesTC) & 1)) {
+            const int unit = ctrl->meta[s].unit;
+            if (unit < 0) {
+              t_end = ts;
+              did = true;
+            } else {
+              const int k = ctrl->meta[s].k;
+              const bool q_ok = (k != 0) || mbar_test(&ctrl->q_full, uo & 1);
+              if (q_ok) {
+                if (k == 0) ++uo;
+                k_of[s] = k;
+                tc_fence_after();
+                const uint32_t d = tmem + (uint32_t)(ts & 1) * kN;
+                const uint32_t kb = sbase + kOffStages + (uint32_t)s * kStageBytes;
 #pragma unroll 1
-          for (int kk = 0; kk < kD / 16; ++kk) {
-            const uint32_t h = kk >> 2, off = (kk & 3) * 32;
-            const uint64_t a = smem_desc_sw128(sbase + h * kHalf + off, 16, 1024);
-            const uint64_t b = smem_desc_sw128(kb + h * kHalf + off, 16, 1024);
-            mma_ss(d, a, b, kIdescS, kk > 0);
+                for (int kk = 0; kk < kD / 16; ++kk) {
+                  const uint32_t h = kk >> 2, off = (kk & 3) * 32;
+                  const uint64_t a = smem_desc_sw128(sbase + h * kHalf + off, 16, 1024);
+                  const uint64_t b = smem_desc_sw128(kb + h * kHalf + off, 16, 1024);
+                  mma_ss(d, a, b, kIdescS, kk > 0);
+                }
+                mma_commit(&ctrl->s_full[ts & 1]);
+                if (ctrl->meta[s].k == ctrl->meta[s].ntu - 1) mma_commit(&ctrl->q_empty);
+                ++ts;
+                did = true;
+              }
+            }
           }
-          mma_commit(&ctrl->s_full[t & 1]);
-          if (last) mma_commit(&ctrl->q_empty);
         }
-        if (have_prev) {
-          const int tp = t - 1;
-          if (!wait_or_abort(&ctrl->p_full[tp & 1], (tp >> 1) & 1, ctrl, p.err)) break;
+        if (tp < ts && mbar_test(&ctrl->p_full[tp & 1], (tp >> 1) & 1)) {
           tc_fence_after();
           const int sp = tp % kStagesTC;
           const uint32_t pcol = tmem + (uint32_t)(tp & 1) * kN;
           const uint32_t ocol = tmem + kColO + (uint32_t)(tp & 1) * kD;
           const uint32_t vb = sbase + kOffStages + (uint32_t)sp * kStageBytes + 2 * kHalf;
+          const bool first = k_of[sp] < 2;
           // tokens [16kk, 16kk+16): P_hi at packed column 32*(kk/2) + 8*(kk%2),
           // P_lo 16 columns further
 #pragma unroll 1
           for (int kk = 0; kk < kN / 16; ++kk) {
             const uint64_t b = smem_desc_sw128(vb + kk * 2048u, kHalf, 1024);
             const uint32_t a = pcol + 32 * (kk >> 1) + 8 * (kk & 1);
-            mma_ts(ocol, a, b, kIdescPV, !(prev_k < 2 && kk == 0));
+            mma_ts(ocol, a, b, kIdescPV, !(first && kk == 0));
             mma_ts(ocol, a + 16, b, kIdescPV, 1);
           }
           mma_commit(&ctrl->o_full[tp & 1]);
           mma_commit(&ctrl->kv_empty[sp]);
+          ++tp;
+          did = true;
         }
-        if (unit < 0) break;
-        prev_k = k;
-        have_prev = true;
-        ++t;
+        if (did) {
+          idle = 0;
+        } else if (++idle > (1u << 26)) {   // bounded: a stuck pipeline gives up
+          ctrl->abort_flag = 1;
+          raise_err(p.err, SEED_DEVERR_TIMEOUT);
+        } else if (idle > 64) {
+          __nanosleep(32);
+        }
       }
     }
     __syncwarp();
