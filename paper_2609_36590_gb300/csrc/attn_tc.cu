@@ -461,9 +461,11 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
     }
     mbar_init(&ctrl->q_full, 1);
     mbar_init(&ctrl->q_empty, 1);
+    // one arrival per lane quarter that can hold query rows in this launch
+    const int nqa = min(4, (p.G * p.W1 + 31) / 32);
     for (int i = 0; i < 2; ++i) {
       mbar_init(&ctrl->s_full[i], 1);
-      mbar_init(&ctrl->p_full[i], 4);
+      mbar_init(&ctrl->p_full[i], nqa);
       mbar_init(&ctrl->o_full[i], 1);
     }
     for (int i = 0; i < 4; ++i) {
@@ -649,19 +651,21 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
           ++tp;
           did = true;
         }
+        // polls without sleeping (a sleep's wake-up granularity would delay
+        // the next MMA); bounded: a stuck pipeline gives up after ~2^28 polls
         if (did) {
           idle = 0;
-        } else if (++idle > (1u << 26)) {   // bounded: a stuck pipeline gives up
+        } else if (++idle > (1u << 28)) {
           ctrl->abort_flag = 1;
           raise_err(p.err, SEED_DEVERR_TIMEOUT);
-        } else if (idle > 64) {
-          __nanosleep(32);
         }
       }
     }
     __syncwarp();
-  } else if (warp < 8) {
+  } else if (warp < 8 && (warp & 3) < min(4, (p.G * p.W1 + 31) / 32)) {
     // ---------------------------------------------------------- softmax
+    // (warps of lane quarters that no query row of this launch reaches skip
+    // the role altogether, so that they never gate the pipeline)
     // Warps 0-3 take the even tiles of the CTA, warps 4-7 the odd ones; each
     // group keeps its own running max, sum and O accumulator per row.  (The
     // producer and MMA warps sit on the SM sub-partitions of lane quarters 2
@@ -672,7 +676,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
     const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
     const uint32_t ocol = tmem + lane_off + kColO + (uint32_t)par * kD;
     const uint32_t ocol_other = tmem + lane_off + kColO + (uint32_t)(par ^ 1) * kD;
-    const int col = (warp - 4 * par) * 32 + lane;   // column whose V row this thread zeroes
+    const int nqa = min(4, (p.G * p.W1 + 31) / 32);   // lane quarters in use
     const float c2 = p.scale_log2;
     float m_used = -INFINITY, l = 0.f;
     int xcnt = 0;
@@ -716,17 +720,21 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
       }
       // V rows of columns nobody may see are zeroed, so that a probability of
       // 0 never meets a stale or NaN-poisoned row
-      {
-        const bool valid = (col < cm.dcol) ? (col < m.cvalid - m.tile * kN) : (col < cm.dend);
-        if (!valid) {
-          uint8_t* vb = smem + kOffStages + (size_t)s * kStageBytes + 2 * kHalf;
+      if (m.cvalid - m.tile * kN < kN || cm.dcol < kN) {
+        uint8_t* vb = smem + kOffStages + (size_t)s * kStageBytes + 2 * kHalf;
+        bool wrote = false;
+#pragma unroll 1
+        for (int col = q4 * 32 + lane; col < kN; col += 32 * nqa) {
+          const bool valid = (col < cm.dcol) ? (col < m.cvalid - m.tile * kN) : (col < cm.dend);
+          if (valid) continue;
 #pragma unroll 1
           for (int ch = 0; ch < 8; ++ch) {
             *reinterpret_cast<uint4*>(vb + col * 128 + ch * 16) = make_uint4(0, 0, 0, 0);
             *reinterpret_cast<uint4*>(vb + kHalf + col * 128 + ch * 16) = make_uint4(0, 0, 0, 0);
           }
-          fence_proxy_async_smem();
+          wrote = true;
         }
+        if (wrote) fence_proxy_async_smem();
       }
       // this group's previous PV must be done before its O is rescaled
       if (own > 0 && !wait_or_abort(&ctrl->o_full[par], (own - 1) & 1, ctrl, p.err)) break;
