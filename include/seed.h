@@ -55,7 +55,8 @@ typedef enum {
   SEED_ERR_RANGE = 3,         /* max_pages / num_pages out of range            */
   SEED_ERR_UNSUPPORTED = 4,   /* head_dim, group size or page_size not built   */
   SEED_ERR_CUDA = 5,          /* a CUDA runtime call failed (launch error)     */
-  SEED_ERR_WORKSPACE = 6      /* workspace too small or misaligned             */
+  SEED_ERR_WORKSPACE = 6,     /* workspace too small or misaligned             */
+  SEED_ERR_SCRATCH_LIMIT = 7  /* problem too large for the built-in scratch    */
 } seed_status_t;
 
 /* Device error bits (OR-ed into *err_flag). */
@@ -189,6 +190,43 @@ seed_status_t seed_accept_commit(int32_t batch, int32_t kmax, const int32_t* dra
                                  int32_t page_size, int32_t* ctx_lens, int32_t* accepted,
                                  int32_t* tokens, int32_t* committed_slots,
                                  int32_t* err_flag, void* stream);
+
+/* ------------------------------------------------------------------------
+ * Library convenience with no counterpart in the paper: verify attention
+ * without a caller-provided workspace.
+ *
+ * seed_verify_attn_noalloc computes exactly what seed_verify_attn computes,
+ * with the same arguments minus ws / ws_bytes. Its workspace is a scratch
+ * array of SEED_NOALLOC_SCRATCH_BYTES built into the library (one per
+ * device), so neither the caller nor the library allocates device memory.
+ * It is meant for callers that cannot provide device memory: a plain C host
+ * with no allocator of its own to expose, or a server that has handed all
+ * free HBM to its KV page pool.
+ *
+ *   - Size limit: the call returns SEED_ERR_SCRATCH_LIMIT and launches
+ *     nothing when seed_workspace_bytes(cfg, batch) exceeds
+ *     SEED_NOALLOC_SCRATCH_BYTES.
+ *   - Set-up: the first call on a device, with that device current, resolves
+ *     the scratch's device address (this can load the library's module on
+ *     the device) and caches it. Make that first call before any stream
+ *     capture begins.
+ *   - Zeroing: each call clears the scratch's counters on `stream` before its
+ *     kernels (one small memset), so the caller never zeroes anything, and a
+ *     call after a device error starts clean.
+ *   - Concurrency: calls on one device that overlap in time (different
+ *     streams, or host threads with no ordering between them) share the
+ *     scratch and RACE. Serialise them: one stream, or events between them.
+ *   - Errors: as seed_verify_attn, plus SEED_ERR_SCRATCH_LIMIT, and
+ *     SEED_ERR_CUDA when the device or the scratch address cannot be
+ *     obtained.
+ * ------------------------------------------------------------------------ */
+#define SEED_NOALLOC_SCRATCH_BYTES (32u << 20)
+
+seed_status_t seed_verify_attn_noalloc(const seed_cfg_t* cfg, int32_t batch,
+                                       const void* q, const int32_t* n_q,
+                                       seed_kv_t kv, const int32_t* ctx_lens,
+                                       float* out, float* lse,
+                                       int32_t* err_flag, void* stream);
 
 #ifdef __cplusplus
 }

@@ -7,7 +7,9 @@ All arithmetic runs in the library's CUDA kernels; there is no fallback, and
 every entry point fails loudly when the library has not been built.
 
 Entry points carry the C names: seed_workspace_bytes, seed_draft_kv_append,
-seed_draft_attn, seed_kv_append, seed_verify_attn, seed_accept_commit.
+seed_draft_attn, seed_kv_append, seed_verify_attn, seed_accept_commit, and
+seed_verify_attn_noalloc (verify attention on the library's built-in scratch,
+for callers that cannot provide a workspace).
 """
 
 from __future__ import annotations
@@ -22,6 +24,8 @@ _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "libseed.so")
 
 SEED_OK = 0
+SEED_ERR_SCRATCH_LIMIT = 7
+NOALLOC_SCRATCH_BYTES = 32 << 20   # SEED_NOALLOC_SCRATCH_BYTES of seed.h
 DEVERR = {1: "ctx_len", 2: "draft_len", 4: "n_q", 8: "page", 16: "k_b", 32: "workspace",
           64: "timeout"}
 MAX_KMAX = 16
@@ -50,6 +54,8 @@ _SIGS = {
     "seed_verify_attn": (_I, [ctypes.POINTER(_Cfg), _I, _P, _P, _KV, _P, _P, _P, _P,
                               ctypes.c_size_t, _P, _P]),
     "seed_accept_commit": (_I, [_I, _I, _P, _P, _P, _P, _I, _I, _P, _P, _P, _P, _P, _P]),
+    "seed_verify_attn_noalloc": (_I, [ctypes.POINTER(_Cfg), _I, _P, _P, _KV, _P, _P, _P, _P,
+                                      _P]),
 }
 
 
@@ -217,6 +223,25 @@ def seed_verify_attn(cfg: SeedConfig, q, n_q, kv: PagedKV, ctx_lens, out, lse, w
         _t(out, torch.float32, (B, W, cfg.hq, cfg.head_dim), "out"),
         _t(lse, torch.float32, (B, W, cfg.hq), "lse") if lse is not None else None,
         _t(ws, torch.uint8, None, "ws"), ws.numel(),
+        _t(err, torch.int32, (1,), "err"), _stream(stream)))
+
+
+def seed_verify_attn_noalloc(cfg: SeedConfig, q, n_q, kv: PagedKV, ctx_lens, out, lse, err,
+                             stream=None) -> None:
+    """seed_verify_attn without a workspace argument: the library uses its
+    built-in per-device scratch. Calls that overlap in time on one device race
+    on that scratch; issue them on one stream."""
+    B = q.shape[0]
+    c = cfg.c()
+    W = cfg.kmax + 1
+    _check(_lib.seed_verify_attn_noalloc(
+        ctypes.byref(c), B,
+        _t(q, torch.bfloat16, (B, W, cfg.hq, cfg.head_dim), "q"),
+        _t(n_q, torch.int32, (B,), "n_q"),
+        _kv_checked(cfg, kv, B),
+        _t(ctx_lens, torch.int32, (B,), "ctx_lens"),
+        _t(out, torch.float32, (B, W, cfg.hq, cfg.head_dim), "out"),
+        _t(lse, torch.float32, (B, W, cfg.hq), "lse") if lse is not None else None,
         _t(err, torch.int32, (1,), "err"), _stream(stream)))
 
 

@@ -145,6 +145,8 @@ const char* seed_status_string(seed_status_t s) {
     case SEED_ERR_UNSUPPORTED: return "head_dim, group size or page_size not supported";
     case SEED_ERR_CUDA: return "CUDA launch failed";
     case SEED_ERR_WORKSPACE: return "workspace too small or misaligned";
+    case SEED_ERR_SCRATCH_LIMIT:
+      return "problem needs more workspace than the built-in scratch holds";
   }
   return "unknown status";
 }
