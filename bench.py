@@ -73,6 +73,43 @@ def round_bytes(wl, lens: np.ndarray, k_b: np.ndarray, n_layers: int) -> dict:
                 accept=accept, total=draft + verify + accept)
 
 
+# ------------------------------------------------------------------ ncu traffic
+# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) of one attention
+# launch from an ncu capture of `bench.py --profile <kind> --workload <n>`
+# (one launch on the workload's two decoder layers), with the algorithmic bytes
+# of that launch and a hash of the kernel's sources at capture time.  The
+# reported traffic is scaled to the timed launches by their algorithmic bytes,
+# and is null once the kernel's sources differ from the captured ones.
+NCU_TRAFFIC = {
+    (3, "verify"): {"kernel": "attn_tc_kernel", "sources": "62a452f18ef2669c",
+                    "dram_bytes": 166086656 + 10738432, "alg_bytes": 165939200},
+    (3, "draft"): {"kernel": "attn_tc_kernel", "sources": "62a452f18ef2669c",
+                   "dram_bytes": 165008384 + 10237696, "alg_bytes": 164096000},
+}
+
+KERNEL_SOURCES = {
+    "attn_tc_kernel": ["attn_tc.cu", "tc.cuh", "common.cuh", "kernels.h"],
+    "decode_attn_kernel": ["decode_attn.cu", "common.cuh", "kernels.h"],
+}
+
+
+def kernel_source_hash(name: str) -> str:
+    import hashlib
+    h = hashlib.sha256()
+    for f in KERNEL_SOURCES[name]:
+        with open(os.path.join(ROOT, "paper_2609_36590_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def ncu_traffic(wl, kind: str, alg_bytes: float):
+    rec = NCU_TRAFFIC.get((wl.index, kind))
+    name = attn_kernel_name(wl)
+    if rec is None or rec["kernel"] != name or rec["sources"] != kernel_source_hash(name):
+        return None
+    return round(rec["dram_bytes"] * alg_bytes / rec["alg_bytes"])
+
+
 # ------------------------------------------------------------------ clocks
 class ClockSampler:
     QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
@@ -165,15 +202,19 @@ def run_seed(args, rank, world, device):
     wl = WORKLOADS[args.workload]
     W, K = args.warmup, args.steps
     torch.cuda.set_device(device)
-    dw = DeviceWorkload(wl, device=device, rounds=W + K + 1)
+    # rounds [W, W+K) are the timed steps; rounds [W+K, W+2K) repeat the same
+    # kind of step with timing events around every attention launch (those
+    # events serialise the stream, so they stay out of the timed steps)
+    n_rounds = W + 2 * K
+    dw = DeviceWorkload(wl, device=device, rounds=n_rounds + 1)
     stream = torch.cuda.Stream(device=device)
 
     # host bookkeeping of lengths (the planned acceptance is what accept returns)
     lens = [dw.lens0.astype(np.int64)]
-    for r in range(W + K):
+    for r in range(n_rounds):
         _, n_plan, _, _ = gen.round_plan(wl, r)
         lens.append(lens[-1] + n_plan + 1)
-    for r in range(W + K):
+    for r in range(n_rounds):
         dw.round_inputs(r)
 
     # round 0 runs eagerly (sets launch attributes); later rounds replay graphs
@@ -182,16 +223,20 @@ def run_seed(args, rank, world, device):
     stream.synchronize()
     assert int(dw.err.item()) == 0, "device error flag raised in warm-up"
 
-    graphs = {}
-    for r in range(1, W + K):
+    graphs, timers = {}, {}
+    for r in range(1, n_rounds):
         ins = dw.round_inputs(r)
+        marks = None
+        if r >= W + K:
+            timers[r] = AttnTimer()
+            marks = timers[r].marks()
         gd, gv, ga = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
         with torch.cuda.graph(gd, stream=stream):
             for i in range(1, ins["steps"] + 1):
-                dw.draft_step(ins, i)
+                dw.draft_step(ins, i, marks=marks)
         with torch.cuda.graph(gv, stream=stream):
             for l in dw.layers:
-                dw.verify_layer(ins, l)
+                dw.verify_layer(ins, l, marks=marks)
         with torch.cuda.graph(ga, stream=stream):
             dw.accept(ins)
         graphs[r] = (gd, gv, ga)
@@ -222,10 +267,16 @@ def run_seed(args, rank, world, device):
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
+    # the kernel-timing rounds
+    with torch.cuda.stream(stream):
+        for t in range(K):
+            for g in graphs[W + K + t]:
+                g.replay()
+    stream.synchronize()
     clocks = sampler.stop() if sampler else None
     assert int(dw.err.item()) == 0, "device error flag raised in timed rounds"
     got_lens = dw.ctx_lens.cpu().numpy()
-    assert (got_lens == lens[W + K]).all(), "accepted lengths diverged from the plan"
+    assert (got_lens == lens[n_rounds]).all(), "accepted lengths diverged from the plan"
 
     t_round = [ev[t][0].elapsed_time(ev[t][3]) for t in range(K)]
     t_draft = [ev[t][0].elapsed_time(ev[t][1]) for t in range(K)]
@@ -236,38 +287,121 @@ def run_seed(args, rank, world, device):
     total_bytes = sum(b["total"] for b in byt)
     steps_per_round = [int(gen.round_plan(wl, W + t)[0].max()) for t in range(K)]
 
-    # dominant kernel: verify attention alone, all layers back to back
-    ins = dw.round_inputs(W + K - 1)
-    gk = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(gk, stream=stream):
-        for l in dw.layers:
-            q, _, _ = ins["verify"][l]
-            import paper_2609_36590_gb300 as seed
-            seed.seed_verify_attn(dw.cfg, q, ins["n_q"], dw.kv[l], dw.ctx_lens, dw.out_v,
-                                  dw.lse_v, dw.ws, dw.err)
-    for _ in range(2):
-        gk.replay()
-    k0, k1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    reps = max(3, K)
-    with torch.cuda.stream(stream):
-        k0.record(stream)
-        for _ in range(reps):
-            gk.replay()
-        k1.record(stream)
-    stream.synchronize()
-    cur = got_lens.astype(np.int64)
-    kbytes = round_bytes(wl, cur, ins["k_b_np"], len(dw.layers))["verify_attn"]
-    per_launch_s = k0.elapsed_time(k1) / 1e3 / (reps * len(dw.layers))
-    k_gbs = kbytes / len(dw.layers) / per_launch_s / 1e9
+    # attention kernels: every launch of the kernel-timing rounds, timed by
+    # the events recorded around it inside the round graphs
+    kern = {}
+    for kind in ("verify", "draft"):
+        nbytes = secs = launches = 0
+        for r in range(W + K, n_rounds):
+            k_b = gen.round_plan(wl, r)[0]
+            for key, ms in timers[r].durations(kind):
+                nbytes += attn_call_bytes(wl, kind, key, lens[r], k_b)
+                secs += ms / 1e3
+                launches += 1
+        kern[kind] = dict(gbs=nbytes / secs / 1e9, us=secs / launches * 1e6,
+                          bytes=nbytes / launches, launches=launches)
 
     res = dict(total_ms=total_ms, total_bytes=total_bytes, t_round=t_round, t_draft=t_draft,
-               t_verify=t_verify, steps_per_round=steps_per_round, clocks=clocks,
-               kernel_gbs=k_gbs, kernel_us=per_launch_s * 1e6,
-               kernel_bytes=kbytes / len(dw.layers), n_launches=count_launches(wl, steps_per_round,
-                                                                               len(dw.layers)))
+               t_verify=t_verify, steps_per_round=steps_per_round, clocks=clocks, kern=kern,
+               n_launches=count_launches(wl, steps_per_round, len(dw.layers)))
     if not args.no_e2e:
         res["e2e"] = run_e2e(dw, wl, stream, W, K, lens)
     return res
+
+
+class AttnTimer:
+    """CUDA events recorded around each attention call while a round graph is
+    captured.  They are external events, so the graph holds real event-record
+    nodes and every replay stamps them on the launching stream."""
+
+    def __init__(self):
+        self.calls = []
+
+    def marks(self):
+        import torch
+
+        def before(kind, key):
+            e = torch.cuda.Event(enable_timing=True, external=True)
+            e.record()
+            self.calls.append([kind, key, e, None])
+
+        def after(kind, key):
+            e = torch.cuda.Event(enable_timing=True, external=True)
+            e.record()
+            self.calls[-1][3] = e
+
+        return before, after
+
+    def durations(self, kind):
+        return [(key, a.elapsed_time(b)) for k, key, a, b in self.calls if k == kind]
+
+
+def attn_call_bytes(wl, kind, key, lens, k_b) -> int:
+    """Algorithmic bytes of one attention launch (one layer): every visible K/V
+    row once, plus q in and o, lse out for each active query row."""
+    R = wl.row_bytes
+    qo = wl.hq * wl.head_dim * (2 + 4) + wl.hq * 4
+    if kind == "draft":
+        i = key[0]
+        return sum((int(L) + i) * R + qo for L, kb in zip(lens, k_b) if kb >= i)
+    return sum((int(L) + int(kb) + 1) * R + (int(kb) + 1) * qo for L, kb in zip(lens, k_b))
+
+
+def attn_kernel_name(wl) -> str:
+    """The kernel behind seed_draft_attn / seed_verify_attn for this shape: the
+    tensor-core kernel when head_dim is 128 and the query rows of one KV head
+    fit one 128-row tile, else the CUDA-core split-KV kernel."""
+    G = wl.hq // wl.hkv
+    return "attn_tc_kernel" if wl.head_dim == 128 and G * (wl.kmax + 1) <= 128 \
+        else "decode_attn_kernel"
+
+
+def run_profile(args):
+    """--profile draft|verify: the appends of round 0 on the workload's two
+    decoder layers, then `--reps` launches of one attention kind alternating
+    between them (a few hundred MB of KV, above the L2 size).  For ncu captures
+    of one launch (`-k regex:<kernel> -s 2 -c 1`); prints the algorithmic bytes
+    of each launch, no bench value."""
+    import torch
+
+    from paper_2609_36590_gb300 import build
+    build.build()
+    import paper_2609_36590_gb300 as seed
+    from workloads.device import DeviceWorkload
+
+    wl = WORKLOADS[args.workload]
+    torch.cuda.set_device(0)
+    dw = DeviceWorkload(wl, device="cuda:0", layers=list(wl.dec_layers), rounds=2)
+    ins = dw.round_inputs(0)
+    k_b = ins["k_b_np"]
+    lens = dw.lens0
+    dec = list(wl.dec_layers)
+    for l in dec:
+        q, kn, vn = ins["draft"][(1, l)]
+        seed.seed_draft_kv_append(dw.cfg, kn, vn, ins["draft_lens"][0], dw.draft_k[l],
+                                  dw.draft_v[l], dw.err)
+        _, kn, vn = ins["verify"][l]
+        seed.seed_kv_append(dw.cfg, dw.kv[l], kn, vn, ins["n_q"], dw.ctx_lens, dw.err)
+    torch.cuda.synchronize()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.reps + 1)]
+    ev[0].record()
+    for r in range(args.reps):
+        l = dec[r % len(dec)]
+        if args.profile == "draft":
+            dw.draft_attn(ins, 1, l)
+        else:
+            dw.verify_attn(ins, l)
+        ev[r + 1].record()
+    torch.cuda.synchronize()
+    assert int(dw.err.item()) == 0, "device error flag raised"
+    key = (1, dec[0]) if args.profile == "draft" else dec[0]
+    nbytes = attn_call_bytes(wl, args.profile, key, lens, k_b)
+    print(json.dumps({"profile": args.profile, "workload": wl.name,
+                      "kernel": attn_kernel_name(wl),
+                      "sources": kernel_source_hash(attn_kernel_name(wl)),
+                      "alg_bytes_per_launch": nbytes,
+                      "us": [round(ev[i].elapsed_time(ev[i + 1]) * 1e3, 1)
+                             for i in range(args.reps)]}))
 
 
 def count_launches(wl, steps_per_round, n_layers):
@@ -372,7 +506,13 @@ def main():
     ap.add_argument("--impl", default="seed", choices=["seed", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=12.0)
+    ap.add_argument("--profile", choices=["draft", "verify"], default=None,
+                    help="launch one attention kind a few times for an ncu capture")
+    ap.add_argument("--reps", type=int, default=3)
     args = ap.parse_args()
+    if args.profile:
+        run_profile(args)
+        return
     if args.warmup < 1:
         ap.error("--warmup must be >= 1")
 
@@ -423,6 +563,7 @@ def main():
     if rank == 0:
         cpu = oracle_sample(wl, args.cpu_budget) if world == 1 else None
         K = args.steps
+        kv_, kd_ = res["kern"]["verify"], res["kern"]["draft"]
         line = {
             "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
             "steps": K, "warmup": args.warmup, "ms_per_step": total_s * 1e3 / K,
@@ -433,12 +574,21 @@ def main():
             "draft_step_us": 1e3 * sum(res["t_draft"]) / sum(res["steps_per_round"]),
             "verify_step_us": 1e3 * statistics.mean(res["t_verify"]),
             "round_us": 1e3 * statistics.mean(res["t_round"]),
-            "roofline": {"bound": "hbm", "kernel": "seed_verify_attn (decode_attn_kernel)",
-                         "achieved": round(res["kernel_gbs"], 1), "peak": peak,
-                         "unit": "GB/s", "frac": round(res["kernel_gbs"] / peak, 3),
-                         "peak_kind": peak_kind, "traffic": None,
-                         "bytes_per_launch": res["kernel_bytes"],
-                         "us_per_launch": round(res["kernel_us"], 2)},
+            "roofline": {"bound": "hbm",
+                         "kernel": f"seed_verify_attn ({attn_kernel_name(wl)})",
+                         "achieved": round(kv_["gbs"], 1), "peak": peak,
+                         "unit": "GB/s", "frac": round(kv_["gbs"] / peak, 3),
+                         "peak_kind": peak_kind,
+                         "traffic": ncu_traffic(wl, "verify", kv_["bytes"]),
+                         "bytes_per_launch": round(kv_["bytes"]),
+                         "us_per_launch": round(kv_["us"], 2), "launches": kv_["launches"],
+                         "timing": "CUDA events around every launch of K more rounds"},
+            "draft_attn": {"kernel": f"seed_draft_attn ({attn_kernel_name(wl)})",
+                           "achieved": round(kd_["gbs"], 1),
+                           "frac": round(kd_["gbs"] / peak, 3),
+                           "traffic": ncu_traffic(wl, "draft", kd_["bytes"]),
+                           "bytes_per_launch": round(kd_["bytes"]),
+                           "us_per_launch": round(kd_["us"], 2), "launches": kd_["launches"]},
             "gpu_launches": res["n_launches"],
             "clocks": res["clocks"],
             "cpu_baseline": cpu,

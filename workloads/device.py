@@ -132,23 +132,41 @@ class DeviceWorkload:
         return ins
 
     # ------------------------------------------------------------ one round
-    def draft_step(self, ins: dict, i: int, on_draft=None) -> None:
+    def draft_step(self, ins: dict, i: int, on_draft=None, marks=None) -> None:
+        """marks: optional (before, after) callables run around each attention
+        call, given ("draft", (i, layer)); bench.py records timing events there."""
         for l in self.wl.dec_layers:
             q, kn, vn = ins["draft"][(i, l)]
             dl = ins["draft_lens"][i - 1]
             seed.seed_draft_kv_append(self.cfg, kn, vn, dl, self.draft_k[l], self.draft_v[l], self.err)
-            seed.seed_draft_attn(self.cfg, q, self.kv[l], self.draft_k[l], self.draft_v[l],
-                                 self.ctx_lens, dl, self.out_d, self.lse_d, self.ws, self.err)
+            self.draft_attn(ins, i, l, marks)
             if on_draft is not None:
                 on_draft(i, l, self.out_d, self.lse_d)
 
-    def verify_layer(self, ins: dict, l: int, on_verify=None) -> None:
+    def draft_attn(self, ins: dict, i: int, l: int, marks=None) -> None:
+        q = ins["draft"][(i, l)][0]
+        if marks:
+            marks[0]("draft", (i, l))
+        seed.seed_draft_attn(self.cfg, q, self.kv[l], self.draft_k[l], self.draft_v[l],
+                             self.ctx_lens, ins["draft_lens"][i - 1], self.out_d, self.lse_d,
+                             self.ws, self.err)
+        if marks:
+            marks[1]("draft", (i, l))
+
+    def verify_layer(self, ins: dict, l: int, on_verify=None, marks=None) -> None:
         q, kn, vn = ins["verify"][l]
         seed.seed_kv_append(self.cfg, self.kv[l], kn, vn, ins["n_q"], self.ctx_lens, self.err)
-        seed.seed_verify_attn(self.cfg, q, ins["n_q"], self.kv[l], self.ctx_lens, self.out_v,
-                              self.lse_v, self.ws, self.err)
+        self.verify_attn(ins, l, marks)
         if on_verify is not None:
             on_verify(l, self.out_v, self.lse_v)
+
+    def verify_attn(self, ins: dict, l: int, marks=None) -> None:
+        if marks:
+            marks[0]("verify", l)
+        seed.seed_verify_attn(self.cfg, ins["verify"][l][0], ins["n_q"], self.kv[l],
+                              self.ctx_lens, self.out_v, self.lse_v, self.ws, self.err)
+        if marks:
+            marks[1]("verify", l)
 
     def accept(self, ins: dict) -> None:
         seed.seed_accept_commit(self.wl.kmax, ins["draft_ids"], ins["target_ids"], ins["k_b"],
