@@ -29,11 +29,13 @@
 // query may see (past the sequence end, unfilled page slots) are zeroed in
 // shared memory before PV so that stale or poisoned rows contribute nothing.
 //
-// Work: units of `tpu` tiles of one (b, g) are handed out by an atomic
-// counter, full-size units first and ragged ones last.  Units of the same
-// (b, g) leave normalised partials and log2-sum-exps; per TMEM lane quarter
-// the last warp to finish merges them in unit order, so results are
-// deterministic.
+// Work: the launch's tiles, ordered by (sequence, KV head, tile), are cut
+// into one contiguous range per CTA of (almost) equal length.  A CTA's range
+// covers whole (b, g) pairs, whose outputs it writes directly, and at most
+// two pieces of pairs shared with its neighbours; for those it leaves a
+// normalised partial and its log2-sum-exps in one of its two record slots.
+// A second, small kernel merges the pieces of every shared pair in range
+// order, so results are deterministic and no CTA ever waits for another.
 //
 // Warp roles (384 threads): warps 0-7 softmax / epilogue (two groups of four,
 // one warp per TMEM lane quarter), warp 10 TMA producer and scheduler, warp 11
@@ -76,7 +78,7 @@ constexpr uint32_t kIdescS = idesc_bf16_f32(128, kN, 0, 0);     // K-major A and
 constexpr uint32_t kIdescPV = idesc_bf16_f32(128, kD, 0, 1);    // B (V) MN-major
 
 struct TileMeta {
-  int32_t unit;        // < 0: no more tiles
+  int32_t unit;        // < 0: no more tiles (else: index of the piece in the CTA)
   int32_t b, g;
   int32_t tile;        // tile index within the sequence
   int32_t k, ntu;      // tile index within the unit; tiles in the unit
@@ -84,10 +86,8 @@ struct TileMeta {
   int32_t ncp;         // cache pages of the sequence
   int32_t cvalid;      // cache rows that exist (L, or L + n_q for verify)
   int32_t lim0;        // query j sees cache positions <= lim0 + j
-  int32_t rec0;        // first partial record of the (b, g) pair
-  int32_t chunk;       // unit index within the pair
-  int32_t nunits;      // units of the pair
-  int32_t pad[2];
+  int32_t slot;        // partial record of this piece, or -1: the whole pair
+  int32_t pad[4];
 };
 
 struct Ctrl {
@@ -153,99 +153,97 @@ __device__ __forceinline__ SeqT seq_of(const AttnTcParams& p, int b) {
   return s;
 }
 
-struct Plan {
-  int tpu, full_total, units;
-};
+// ------------------------------------------------------------- partition
+// Tiles of the launch: T = hkv * sum_b tiles(b).  CTA c of N takes the tiles
+// [start(c), start(c+1)) with start(c) = floor(c T / N) when T >= N (every
+// range non-empty), else start(c) = min(c, T) (one tile each for the first T
+// CTAs), so that the CTAs holding one pair are always consecutive.
+__device__ __forceinline__ long long range_start(long long T, int c, int N) {
+  return T >= N ? T * c / N : min((long long)c, T);
+}
 
-__device__ __noinline__ Plan make_plan(const AttnTcParams& p, int lane) {
+// The CTA whose range holds tile x (0 <= x < T).
+__device__ __forceinline__ int cta_of(long long x, long long T, int N) {
+  return T >= N ? (int)(((x + 1) * N - 1) / T) : (int)x;
+}
+
+// Warp-cooperative: T.
+__device__ __noinline__ long long total_tiles(const AttnTcParams& p, int lane) {
   long long tot = 0;
   for (int b = lane; b < p.B; b += 32) tot += seq_of(p, b).tiles;
   for (int o = 16; o; o >>= 1) tot += __shfl_xor_sync(kFull, tot, o);
-  tot *= p.hkv;
-  Plan pl;
-  pl.tpu = (int)max(1LL, (tot + p.target_units - 1) / p.target_units);
-  int full = 0, part = 0;
-  for (int b = lane; b < p.B; b += 32) {
-    const int t = seq_of(p, b).tiles;
-    full += p.hkv * (t / pl.tpu);
-    part += p.hkv * ((t % pl.tpu) != 0);
-  }
-  for (int o = 16; o; o >>= 1) {
-    full += __shfl_xor_sync(kFull, full, o);
-    part += __shfl_xor_sync(kFull, part, o);
-  }
-  pl.full_total = full;
-  pl.units = full + part;
-  return pl;
+  return tot * p.hkv;
 }
 
-struct UnitInfo {
-  int b, g, chunk, t0, t1, rec0, nunits;
-  SeqT s;
+// A window of 32 sequences [wb, wb + 32); lane i holds sequence wb + i.
+struct SeqWin {
+  int wb;
+  SeqT mine;
 };
 
-// Warp-cooperative: map dense unit index u to (b, g, chunk).  Units
-// [0, full_total) are the full-size units (tpu tiles) of all pairs, the rest
-// the ragged last units.  Record indices follow (b, g, chunk) order.
-__device__ __noinline__ UnitInfo lookup_unit(const AttnTcParams& p, const Plan& pl, int u,
-                                             int lane) {
-  const bool full_phase = u < pl.full_total;
-  const int target = full_phase ? u : u - pl.full_total;
-  int base1 = 0, base2 = 0;
-  UnitInfo ui{};
-  ui.b = -1;
-  for (int start = 0; start < p.B; start += 32) {
-    const int b = start + lane;
-    int a1 = 0, a2 = 0;
-    SeqT st{};
-    if (b < p.B) {
-      st = seq_of(p, b);
-      const int F = st.tiles / pl.tpu, P = (st.tiles % pl.tpu) != 0;
-      a1 = p.hkv * (full_phase ? F : P);
-      a2 = p.hkv * (F + P);
-    }
-    int s1 = a1, s2 = a2;
+__device__ __forceinline__ SeqT seq_or_empty(const AttnTcParams& p, int b) {
+  return b < p.B ? seq_of(p, b) : SeqT{};
+}
+
+__device__ __forceinline__ SeqT win_get(const SeqWin& w, int b) {
+  const int src = b - w.wb;
+  SeqT s;
+  s.nq = __shfl_sync(kFull, w.mine.nq, src);
+  s.nd = __shfl_sync(kFull, w.mine.nd, src);
+  s.ncp = __shfl_sync(kFull, w.mine.ncp, src);
+  s.cvalid = __shfl_sync(kFull, w.mine.cvalid, src);
+  s.lim0 = __shfl_sync(kFull, w.mine.lim0, src);
+  s.tiles = __shfl_sync(kFull, w.mine.tiles, src);
+  s.bad = 0;
+  return s;
+}
+
+// Warp-cooperative: the (sequence b, KV head g, tile t) of tile x < T, with
+// the window that holds b.
+__device__ __noinline__ void locate(const AttnTcParams& p, long long x, int lane, SeqWin& w,
+                                    int& b, int& g, int& t) {
+  long long base = 0;
+  for (w.wb = 0; w.wb < p.B; w.wb += 32) {
+    w.mine = seq_or_empty(p, w.wb + lane);
+    const long long a = (long long)p.hkv * w.mine.tiles;
+    long long inc = a;
     for (int o = 1; o < 32; o <<= 1) {
-      const int t1 = __shfl_up_sync(kFull, s1, o), t2 = __shfl_up_sync(kFull, s2, o);
-      if (lane >= o) {
-        s1 += t1;
-        s2 += t2;
-      }
+      const long long v = __shfl_up_sync(kFull, inc, o);
+      if (lane >= o) inc += v;
     }
-    const bool hit = b < p.B && a1 > 0 && base1 + s1 - a1 <= target && target < base1 + s1;
-    const unsigned m = __ballot_sync(kFull, hit);
-    if (m) {
+    const long long tot = __shfl_sync(kFull, inc, 31);
+    if (x < base + tot) {
+      const unsigned m = __ballot_sync(kFull, base + inc - a <= x && x < base + inc);
       const int src = __ffs(m) - 1;
-      const int pre1 = base1 + __shfl_sync(kFull, s1 - a1, src);
-      const int pre2 = base2 + __shfl_sync(kFull, s2 - a2, src);
-      ui.b = start + src;
-      ui.s.nq = __shfl_sync(kFull, st.nq, src);
-      ui.s.nd = __shfl_sync(kFull, st.nd, src);
-      ui.s.ncp = __shfl_sync(kFull, st.ncp, src);
-      ui.s.cvalid = __shfl_sync(kFull, st.cvalid, src);
-      ui.s.lim0 = __shfl_sync(kFull, st.lim0, src);
-      ui.s.tiles = __shfl_sync(kFull, st.tiles, src);
-      const int F = ui.s.tiles / pl.tpu, P = (ui.s.tiles % pl.tpu) != 0;
-      ui.nunits = F + P;
-      const int r = target - pre1;
-      if (full_phase) {
-        ui.g = r / F;
-        ui.chunk = r - ui.g * F;
-        ui.t0 = ui.chunk * pl.tpu;
-        ui.t1 = ui.t0 + pl.tpu;
-      } else {
-        ui.g = r;
-        ui.chunk = F;
-        ui.t0 = F * pl.tpu;
-        ui.t1 = ui.s.tiles;
-      }
-      ui.rec0 = pre2 + ui.g * ui.nunits;
-      return ui;
+      const long long r = x - base - __shfl_sync(kFull, inc - a, src);
+      const int tiles = __shfl_sync(kFull, w.mine.tiles, src);
+      b = w.wb + src;
+      g = (int)(r / tiles);
+      t = (int)(r - (long long)g * tiles);
+      return;
     }
-    base1 += __shfl_sync(kFull, s1, 31);
-    base2 += __shfl_sync(kFull, s2, 31);
+    base += tot;
   }
-  return ui;
+  b = p.B;
+  g = t = 0;
+}
+
+// Warp-cooperative: the next sequence after b with at least one tile (p.B if
+// none), moving the window forward as needed.
+__device__ __noinline__ void next_seq(const AttnTcParams& p, int lane, SeqWin& w, int& b) {
+  for (;;) {
+    const unsigned m = __ballot_sync(kFull, w.mine.tiles > 0 && w.wb + lane > b);
+    if (m) {
+      b = w.wb + __ffs(m) - 1;
+      return;
+    }
+    w.wb += 32;
+    if (w.wb >= p.B) {
+      b = p.B;
+      return;
+    }
+    w.mine = seq_or_empty(p, w.wb + lane);
+  }
 }
 
 // ------------------------------------------------------------- the kernel
@@ -253,7 +251,6 @@ __device__ __noinline__ UnitInfo lookup_unit(const AttnTcParams& p, const Plan& 
 // columns c <= lim (c < dcol) and the draft columns dcol <= c < dend.
 struct ColMask {
   int dcol, dend, lim;
-  __device__ __forceinline__ bool vis(int c) const { return (c < dcol) ? (c <= lim) : (c < dend); }
   // bit i set <=> column c0 + i is visible
   __device__ __forceinline__ uint32_t bits(int c0) const {
     const int nc = min(max(min(lim, dcol - 1) - c0 + 1, 0), 32);
@@ -323,16 +320,15 @@ __device__ __forceinline__ float row_p(uint32_t scol, const ColMask& cm, float c
   return (ls[0] + ls[1]) + (ls[2] + ls[3]);
 }
 
-// Epilogue of one unit for one warp's rows (run by the group that processed
-// the unit's last tile): combine the two groups' partial softmax states,
-// normalise, and write the output rows -- or this unit's partial record, in
-// which case the last warp (per pair and lane quarter) to finish merges all
-// records of the pair.  Kept out of line: it runs once per unit and needs
-// more registers than the per-tile loop.
-__device__ __noinline__ void unit_epilogue(const AttnTcParams& p, int b, int g, int nq, int rec0,
-                                           int chunk, int nunits, int row, int q4, int lane,
-                                           uint32_t ocol, uint32_t ocol_other, float m_used,
-                                           float l, float mo, float lo) {
+// Epilogue of one piece for one warp's rows (run by the group that processed
+// the piece's last tile): combine the two groups' partial softmax states,
+// normalise, and write the output rows -- or, for a piece of a pair shared
+// with other CTAs, this piece's partial record (same row-major layout:
+// [row][d], then the per-row log2-sum-exp) for the merge kernel.  Kept out of
+// line: it runs once per piece and needs more registers than the tile loop.
+__device__ __noinline__ void unit_epilogue(const AttnTcParams& p, int b, int g, int nq, int slot,
+                                           int row, uint32_t ocol, uint32_t ocol_other,
+                                           float m_used, float l, float mo, float lo) {
   const int Rmax = p.G * p.W1;
   const int R = nq * p.G;
   const int j = row / p.G;
@@ -343,12 +339,11 @@ __device__ __noinline__ void unit_epilogue(const AttnTcParams& p, int b, int g, 
   const float inv = (Ls > 0.f) ? 1.f / Ls : 0.f;
   const float lse2 = (Ls > 0.f) ? M + log2f(Ls) : -INFINITY;
   const bool use_other = __any_sync(kFull, lo > 0.f);
-  const int REC = Rmax * (kD + 1);
   const bool real = row < R;
   const int qh = g * p.G + (row - j * p.G);
   const size_t orow = ((size_t)b * p.W1 + j) * p.hq + qh;   // [b, j, head]
-  float* dst_out = p.out + orow * kD;
-  float* rec = p.part + (size_t)(rec0 + chunk) * REC;
+  float* rec = p.part + (size_t)max(slot, 0) * Rmax * (kD + 1);
+  float* dst = slot < 0 ? p.out + orow * kD : rec + (size_t)row * kD;
 #pragma unroll 1
   for (int c = 0; c < kD / 16; ++c) {
     uint32_t ra[16], rb[16];
@@ -363,78 +358,124 @@ __device__ __noinline__ void unit_epilogue(const AttnTcParams& p, int b, int g, 
       v[i] = x * inv;
     }
     if (real) {
-      // final output row, or this unit's partial record (same
-      // row-major layout: [row][d] then the per-row log2-sum-exp)
-      float4* dp = reinterpret_cast<float4*>(
-          (nunits == 1 ? dst_out : rec + (size_t)row * kD) + c * 16);
+      float4* dp = reinterpret_cast<float4*>(dst + c * 16);
 #pragma unroll
       for (int i = 0; i < 4; ++i)
         dp[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
     }
   }
-  if (nunits == 1) {
-    if (real && p.lse != nullptr) p.lse[orow] = lse2 * kLn2;
-  } else {
-    if (real) rec[(size_t)kD * Rmax + row] = lse2;
-    __threadfence();
-    __syncwarp();
-    int lastw = 0;
-    if (lane == 0)
-      lastw = atomicAdd(&p.counters[(b * p.hkv + g) * 4 + q4], 1) == nunits - 1;
-    lastw = __shfl_sync(kFull, lastw, 0);
-    if (lastw) {
-      // this warp merges its rows over all units of the pair
-      __threadfence();
-      if (real) {
-        const float* base = p.part + (size_t)rec0 * REC;
-        // log2-sum-exps of all units first (independent loads), then the rows
-        // in 32-column slices with up to 4 units' loads in flight at a time
-        float Mx = -INFINITY;
-        for (int c = 0; c < nunits; ++c)
-          Mx = fmaxf(Mx, __ldcg(base + (size_t)c * REC + (size_t)kD * Rmax + row));
-        float S = 0.f;
-        for (int c = 0; c < nunits; ++c) {
-          const float lc = __ldcg(base + (size_t)c * REC + (size_t)kD * Rmax + row);
-          S += (lc == -INFINITY) ? 0.f : ex2_approx(lc - Mx);
-        }
-        const float invS = 1.f / S;
-#pragma unroll 1
-        for (int d0 = 0; d0 < kD; d0 += 32) {
-          float4 acc[8];
+  if (real) {
+    if (slot >= 0)
+      rec[(size_t)kD * Rmax + row] = lse2;
+    else if (p.lse != nullptr)
+      p.lse[orow] = lse2 * kLn2;
+  }
+}
+
+// Merge of the pieces of pair (b, g) = (blockIdx.x / hkv, blockIdx.x % hkv)
+// when the pair's tiles span several CTAs of the attention kernel: the
+// pieces' records are combined with weights 2^(lse_i - M) / sum, in range
+// order.  Pairs that one CTA finished alone return at once.  Loads are
+// issued kMergeBatch pieces at a time so that their latencies overlap.
+constexpr int kMergeThreads = 256;
+constexpr int kMergeBatch = 8;
+
+__global__ void __launch_bounds__(kMergeThreads) attn_merge_kernel(const AttnTcParams p) {
+  __shared__ long long red[2][kMergeThreads / 32];
+  __shared__ float s_m[128], s_inv[128];
+  const int pair = blockIdx.x;
+  const int b = pair / p.hkv, g = pair - b * p.hkv;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  long long tot = 0, pre = 0;
+  for (int i = tid; i < p.B; i += kMergeThreads) {
+    const int t = seq_of(p, i).tiles;
+    tot += t;
+    if (i < b) pre += t;
+  }
+  for (int o = 16; o; o >>= 1) {
+    tot += __shfl_xor_sync(kFull, tot, o);
+    pre += __shfl_xor_sync(kFull, pre, o);
+  }
+  if (lane == 0) {
+    red[0][warp] = tot;
+    red[1][warp] = pre;
+  }
+  __syncthreads();
+  tot = pre = 0;
 #pragma unroll
-          for (int i = 0; i < 8; ++i) acc[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 1
-          for (int c0 = 0; c0 < nunits; c0 += 4) {
-            float4 x[4][8];
-            float w[4];
+  for (int w = 0; w < kMergeThreads / 32; ++w) {
+    tot += red[0][w];
+    pre += red[1][w];
+  }
+  const SeqT sq = seq_of(p, b);
+  if (sq.tiles == 0) return;
+  const long long T = tot * p.hkv;
+  const long long P0 = pre * p.hkv + (long long)g * sq.tiles, P1 = P0 + sq.tiles;
+  const int c_lo = cta_of(P0, T, p.nctas), c_hi = cta_of(P1 - 1, T, p.nctas);
+  if (c_lo == c_hi) return;
+  const int nseg = c_hi - c_lo + 1;
+  // the piece of CTA c_lo is its first piece if its range starts with it
+  const int slot_lo = 2 * c_lo + (range_start(T, c_lo, p.nctas) == P0 ? 0 : 1);
+  const int Rmax = p.G * p.W1;
+  const size_t REC = (size_t)Rmax * (kD + 1);
+  const int R = sq.nq * p.G;
+  const float* lse_base = p.part + (size_t)kD * Rmax;    // + slot * REC + row
+  // row statistics: one online pass over the pieces' log2-sum-exps
+  for (int r = tid; r < R; r += kMergeThreads) {
+    float M = -INFINITY, S = 0.f;
+    for (int i0 = 0; i0 < nseg; i0 += kMergeBatch) {
+      float li[kMergeBatch];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-              const int c = c0 + u;
-              const float* rc = base + (size_t)min(c, nunits - 1) * REC;
-              const float lc = __ldcg(rc + (size_t)kD * Rmax + row);
-              w[u] = (c >= nunits || lc == -INFINITY) ? 0.f : ex2_approx(lc - Mx) * invS;
-              const float4* rp = reinterpret_cast<const float4*>(rc + (size_t)row * kD + d0);
-#pragma unroll
-              for (int i = 0; i < 8; ++i) x[u][i] = __ldcg(rp + i);
-            }
-#pragma unroll
-            for (int u = 0; u < 4; ++u)
-#pragma unroll
-              for (int i = 0; i < 8; ++i) {
-                acc[i].x = fmaf(w[u], x[u][i].x, acc[i].x);
-                acc[i].y = fmaf(w[u], x[u][i].y, acc[i].y);
-                acc[i].z = fmaf(w[u], x[u][i].z, acc[i].z);
-                acc[i].w = fmaf(w[u], x[u][i].w, acc[i].w);
-              }
-          }
-          float4* dp = reinterpret_cast<float4*>(dst_out + d0);
-#pragma unroll
-          for (int i = 0; i < 8; ++i) dp[i] = acc[i];
-        }
-        if (p.lse != nullptr) p.lse[orow] = (Mx + log2f(S)) * kLn2;
+      for (int u = 0; u < kMergeBatch; ++u) {
+        const int i = min(i0 + u, nseg - 1);
+        const int slot = i == 0 ? slot_lo : 2 * (c_lo + i);
+        li[u] = (i0 + u < nseg) ? __ldcg(lse_base + slot * REC + r) : -INFINITY;
       }
-      if (lane == 0) p.counters[(b * p.hkv + g) * 4 + q4] = 0;
+#pragma unroll
+      for (int u = 0; u < kMergeBatch; ++u) {
+        if (li[u] == -INFINITY) continue;
+        if (li[u] > M) {
+          S = S * ex2_approx(M - li[u]) + 1.f;
+          M = li[u];
+        } else {
+          S += ex2_approx(li[u] - M);
+        }
+      }
     }
+    s_m[r] = M;
+    s_inv[r] = 1.f / S;
+    const int j = r / p.G;
+    const size_t orow = ((size_t)b * p.W1 + j) * p.hq + g * p.G + (r - j * p.G);
+    if (p.lse != nullptr) p.lse[orow] = (M + log2f(S)) * kLn2;
+  }
+  __syncthreads();
+  for (int item = tid; item < R * (kD / 4); item += kMergeThreads) {
+    const int r = item / (kD / 4), c4 = item - r * (kD / 4);
+    const float M = s_m[r], inv = s_inv[r];
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int i0 = 0; i0 < nseg; i0 += kMergeBatch) {
+      float li[kMergeBatch];
+      float4 x[kMergeBatch];
+#pragma unroll
+      for (int u = 0; u < kMergeBatch; ++u) {
+        const int i = min(i0 + u, nseg - 1);
+        const int slot = i == 0 ? slot_lo : 2 * (c_lo + i);
+        const float* rc = p.part + slot * REC;
+        li[u] = (i0 + u < nseg) ? __ldcg(rc + (size_t)kD * Rmax + r) : -INFINITY;
+        x[u] = __ldcg(reinterpret_cast<const float4*>(rc + (size_t)r * kD) + c4);
+      }
+#pragma unroll
+      for (int u = 0; u < kMergeBatch; ++u) {
+        const float w = (li[u] == -INFINITY) ? 0.f : ex2_approx(li[u] - M) * inv;
+        acc.x = fmaf(w, x[u].x, acc.x);
+        acc.y = fmaf(w, x[u].y, acc.y);
+        acc.z = fmaf(w, x[u].z, acc.z);
+        acc.w = fmaf(w, x[u].w, acc.w);
+      }
+    }
+    const int j = r / p.G;
+    const size_t orow = ((size_t)b * p.W1 + j) * p.hq + g * p.G + (r - j * p.G);
+    reinterpret_cast<float4*>(p.out + orow * kD)[c4] = acc;
   }
 }
 
@@ -496,29 +537,33 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
         tma_prefetch_desc(&tm_dv);
       }
     }
-    const Plan pl = make_plan(p, lane);
     if (blockIdx.x == 0) {
       for (int b = lane; b < p.B; b += 32) {
         const int bad = seq_of(p, b).bad;
         if (bad) raise_err(p.err, bad);
       }
     }
+    // this CTA's range [x, x1) of the launch's tiles
+    const long long T = total_tiles(p, lane);
+    long long x = range_start(T, blockIdx.x, p.nctas);
+    const long long x1 = range_start(T, blockIdx.x + 1, p.nctas);
+    SeqWin win;
+    int b = p.B, g = 0, t0 = 0;
+    if (x < x1) locate(p, x, lane, win, b, g, t0);
     int it = 0, uo = 0;
     bool ok = true;
-    while (ok) {
-      int u = 0;
-      if (lane == 0) u = atomicAdd(&p.sched[0], 1);
-      u = __shfl_sync(kFull, u, 0);
-      if (u >= pl.units) break;
-      const UnitInfo ui = lookup_unit(p, pl, u, lane);
-      if (ui.b < 0) break;
-      for (int t = ui.t0; t < ui.t1 && ok; ++t, ++it) {
+    while (ok && x < x1 && b < p.B) {
+      // one piece: tiles [t0, t1) of pair (b, g)
+      const SeqT sq = win_get(win, b);
+      const int t1 = (int)min((long long)sq.tiles, t0 + (x1 - x));
+      const int slot = (t0 == 0 && t1 == sq.tiles) ? -1 : 2 * (int)blockIdx.x + (uo > 0 ? 1 : 0);
+      for (int t = t0; t < t1 && ok; ++t, ++it) {
         const int s = it % kStagesTC;
         // page ids of this tile, one lane per page
         const int vp = t * kPagesPerTile + (lane & 7);
         int pid = -1;
-        if (lane < kPagesPerTile && vp < ui.s.ncp) {
-          pid = p.page_table[(size_t)ui.b * p.max_pages + vp];
+        if (lane < kPagesPerTile && vp < sq.ncp) {
+          pid = p.page_table[(size_t)b * p.max_pages + vp];
           if (pid < 0 || pid >= p.num_pages) {
             raise_err(p.err, SEED_DEVERR_PAGE);
             pid = -1;
@@ -526,33 +571,31 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
         }
         if (it >= kStagesTC)
           ok = wait_or_abort(&ctrl->kv_empty[s], ((it / kStagesTC) - 1) & 1, ctrl, p.err);
-        if (ok && t == ui.t0 && uo > 0) ok = wait_or_abort(&ctrl->q_empty, (uo - 1) & 1, ctrl, p.err);
+        if (ok && t == t0 && uo > 0) ok = wait_or_abort(&ctrl->q_empty, (uo - 1) & 1, ctrl, p.err);
         if (!ok) break;
         int pids[kPagesPerTile];
 #pragma unroll
         for (int pp = 0; pp < kPagesPerTile; ++pp) pids[pp] = __shfl_sync(kFull, pid, pp);
         if (lane == 0) {
           TileMeta& m = ctrl->meta[s];
-          m.unit = u;
-          m.b = ui.b;
-          m.g = ui.g;
+          m.unit = uo;
+          m.b = b;
+          m.g = g;
           m.tile = t;
-          m.k = t - ui.t0;
-          m.ntu = ui.t1 - ui.t0;
-          m.nq = ui.s.nq;
-          m.nd = ui.s.nd;
-          m.ncp = ui.s.ncp;
-          m.cvalid = ui.s.cvalid;
-          m.lim0 = ui.s.lim0;
-          m.rec0 = ui.rec0;
-          m.chunk = ui.chunk;
-          m.nunits = ui.nunits;
-          if (t == ui.t0) {
+          m.k = t - t0;
+          m.ntu = t1 - t0;
+          m.nq = sq.nq;
+          m.nd = sq.nd;
+          m.ncp = sq.ncp;
+          m.cvalid = sq.cvalid;
+          m.lim0 = sq.lim0;
+          m.slot = slot;
+          if (t == t0) {
             mbar_arrive_expect_tx(&ctrl->q_full, 2u * 128u * (uint32_t)Rmax);
-            tma_load_4d(smem, &tm_q, 0, ui.g * p.G, 0, ui.b, &ctrl->q_full);
-            tma_load_4d(smem + kHalf, &tm_q, 64, ui.g * p.G, 0, ui.b, &ctrl->q_full);
+            tma_load_4d(smem, &tm_q, 0, g * p.G, 0, b, &ctrl->q_full);
+            tma_load_4d(smem + kHalf, &tm_q, 64, g * p.G, 0, b, &ctrl->q_full);
           }
-          const int dslot = ui.s.nd > 0 ? ui.s.ncp - t * kPagesPerTile : -1;   // draft page slot
+          const int dslot = sq.nd > 0 ? sq.ncp - t * kPagesPerTile : -1;   // draft page slot
           uint32_t bytes = 0;
 #pragma unroll
           for (int pp = 0; pp < kPagesPerTile; ++pp)
@@ -565,17 +608,25 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
             if (pids[pp] < 0 && !is_draft) continue;
             const CUtensorMap* mk = is_draft ? &tm_dk : &tm_k;
             const CUtensorMap* mv = is_draft ? &tm_dv : &tm_v;
-            const int w = is_draft ? ui.b : pids[pp];
+            const int w = is_draft ? b : pids[pp];
             const uint32_t off = pp * 2048u;
-            tma_load_4d(st + 0 * kHalf + off, mk, 0, 0, ui.g, w, &ctrl->kv_full[s]);
-            tma_load_4d(st + 1 * kHalf + off, mk, 64, 0, ui.g, w, &ctrl->kv_full[s]);
-            tma_load_4d(st + 2 * kHalf + off, mv, 0, 0, ui.g, w, &ctrl->kv_full[s]);
-            tma_load_4d(st + 3 * kHalf + off, mv, 64, 0, ui.g, w, &ctrl->kv_full[s]);
+            tma_load_4d(st + 0 * kHalf + off, mk, 0, 0, g, w, &ctrl->kv_full[s]);
+            tma_load_4d(st + 1 * kHalf + off, mk, 64, 0, g, w, &ctrl->kv_full[s]);
+            tma_load_4d(st + 2 * kHalf + off, mv, 0, 0, g, w, &ctrl->kv_full[s]);
+            tma_load_4d(st + 3 * kHalf + off, mv, 64, 0, g, w, &ctrl->kv_full[s]);
           }
         }
         __syncwarp();
       }
       ++uo;
+      x += t1 - t0;
+      if (x >= x1) break;
+      // the range goes on with the next pair
+      t0 = 0;
+      if (++g == p.hkv) {
+        g = 0;
+        next_seq(p, lane, win, b);
+      }
     }
     // end markers: one for each softmax parity (the MMA thread stops at the first)
     for (int e = 0; e < 2 && ok; ++e, ++it) {
@@ -785,8 +836,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
             lo = ctrl->xl[q4][lane];
           }
           if (warp_active)
-            unit_epilogue(p, m.b, m.g, m.nq, m.rec0, m.chunk, m.nunits, row, q4, lane, ocol,
-                          ocol_other, m_used, l, mo, lo);
+            unit_epilogue(p, m.b, m.g, m.nq, m.slot, row, ocol, ocol_other, m_used, l, mo, lo);
           if (m.ntu >= 2) {
             tc_fence_before();
             __syncwarp();
@@ -804,14 +854,6 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
   if (warp == kWarpMma) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
-  }
-  if (tid == 0) {
-    __threadfence();
-    if (atomicAdd(&p.sched[1], 1) == (int)gridDim.x - 1) {
-      p.sched[0] = 0;
-      p.sched[1] = 0;
-      __threadfence();
-    }
   }
 }
 
@@ -854,7 +896,7 @@ bool attn_tc_supported(int head_dim, int group, int w1) {
   return head_dim == kD && group * w1 <= 128;
 }
 
-int attn_tc_target_units() { return std::min(2 * device_sm_count(), kTcUnitsCap); }
+int attn_tc_ctas() { return std::min(device_sm_count(), kTcMaxCtas); }
 
 cudaError_t launch_attn_tc(const AttnTcParams& prm, const void* q, const void* k_cache,
                            const void* v_cache, const void* draft_k, const void* draft_v,
@@ -900,14 +942,15 @@ cudaError_t launch_attn_tc(const AttnTcParams& prm, const void* q, const void* k
     if (e != cudaSuccess) return e;
     g_tc_attr_set.fetch_or(bit, std::memory_order_acq_rel);
   }
-  const int grid = device_sm_count();
-  attn_tc_kernel<<<grid, kThreadsTC, kSmemTC, st>>>(tq, tk, tv, tdk, tdv, prm);
+  attn_tc_kernel<<<prm.nctas, kThreadsTC, kSmemTC, st>>>(tq, tk, tv, tdk, tdv, prm);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  attn_merge_kernel<<<prm.B * prm.hkv, kMergeThreads, 0, st>>>(prm);
   return cudaGetLastError();
 }
 
-size_t attn_tc_part_bound(int32_t batch, int32_t hkv, int32_t group, int32_t w1) {
-  const size_t rmax = (size_t)group * w1;
-  return ((size_t)kTcUnitsCap + (size_t)batch * hkv) * rmax * (kD + 1) * sizeof(float);
+size_t attn_tc_part_bound(int32_t group, int32_t w1) {
+  return 2 * (size_t)kTcMaxCtas * group * w1 * (kD + 1) * sizeof(float);
 }
 
 }  // namespace seedk

@@ -70,7 +70,7 @@ cudaError_t launch_accept(int32_t B, int32_t kmax, const int32_t* draft_ids,
 int device_sm_count();
 
 // Tensor-core draft and verify attention (attn_tc.cu).
-constexpr int kTcUnitsCap = 1024;   // most work units one launch plans
+constexpr int kTcMaxCtas = 256;     // most CTAs of one launch (two record slots each)
 
 struct AttnTcParams {
   const int32_t* page_table;
@@ -80,20 +80,18 @@ struct AttnTcParams {
   const int32_t* aux;         // verify: n_q [B]; draft: draft_lens [B]
   float* out;                 // f32 [B, W1, hq, 128]
   float* lse;                 // f32 [B, W1, hq] or null
-  float* part;                // partial records
-  int32_t* counters;          // [B * hkv * 4] arrival counters (zero between calls)
-  int32_t* sched;             // [2] unit dispenser and finished-CTA count (zero between calls)
+  float* part;                // partial records: two slots per CTA
   int32_t* err;
   int32_t B, hq, hkv, kmax, G;
   int32_t draft;              // 1: draft attention (cache rows + draft scratch rows)
   int32_t W1;                 // query positions per sequence: kmax+1 (verify) or 1 (draft)
-  int32_t target_units;
+  int32_t nctas;              // CTAs of the attention kernel (static tile partition)
   float scale_log2;
 };
 
 bool attn_tc_supported(int head_dim, int group, int w1);
-int attn_tc_target_units();
-size_t attn_tc_part_bound(int32_t batch, int32_t hkv, int32_t group, int32_t w1);
+int attn_tc_ctas();
+size_t attn_tc_part_bound(int32_t group, int32_t w1);
 cudaError_t launch_attn_tc(const AttnTcParams& p, const void* q, const void* k_cache,
                            const void* v_cache, const void* draft_k, const void* draft_v,
                            cudaStream_t st);

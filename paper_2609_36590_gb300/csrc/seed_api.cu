@@ -99,9 +99,8 @@ seed_status_t run_attn_tc(const seed_cfg_t* cfg, int32_t batch, bool draft, cons
   const int G = cfg->hq / cfg->hkv;
   const int W1 = draft ? 1 : cfg->kmax + 1;
   const size_t cb = kSchedBytes + counters_bytes(cfg, batch);
-  const int target = seedk::attn_tc_target_units();
-  const size_t need = cb + ((size_t)target + (size_t)batch * cfg->hkv) * G * W1 *
-                               (cfg->head_dim + 1) * sizeof(float);
+  const int ctas = seedk::attn_tc_ctas();
+  const size_t need = cb + 2 * (size_t)ctas * G * W1 * (cfg->head_dim + 1) * sizeof(float);
   if (ws_bytes < need) return SEED_ERR_WORKSPACE;
   seedk::AttnTcParams p{};
   p.page_table = kv.page_table;
@@ -111,8 +110,6 @@ seed_status_t run_attn_tc(const seed_cfg_t* cfg, int32_t batch, bool draft, cons
   p.aux = aux;
   p.out = out;
   p.lse = lse;
-  p.sched = static_cast<int32_t*>(ws);
-  p.counters = reinterpret_cast<int32_t*>(static_cast<char*>(ws) + kSchedBytes);
   p.part = reinterpret_cast<float*>(static_cast<char*>(ws) + cb);
   p.err = err;
   p.B = batch;
@@ -122,7 +119,7 @@ seed_status_t run_attn_tc(const seed_cfg_t* cfg, int32_t batch, bool draft, cons
   p.G = G;
   p.draft = draft ? 1 : 0;
   p.W1 = W1;
-  p.target_units = target;
+  p.nctas = ctas;
   p.scale_log2 = scale_of(cfg) * 1.4426950408889634f;
   return finish(seedk::launch_attn_tc(p, q, kv.k, kv.v, draft_k, draft_v,
                                       static_cast<cudaStream_t>(stream)));
@@ -157,9 +154,9 @@ size_t seed_workspace_bytes(const seed_cfg_t* cfg, int32_t batch) {
   const int32_t nv_max = batch * (cfg->kmax + 1);
   size_t part = seedk::decode_workspace_bound(nv_max, cfg->hkv, G, cfg->head_dim);
   if (seedk::attn_tc_supported(cfg->head_dim, G, 1))
-    part = std::max(part, seedk::attn_tc_part_bound(batch, cfg->hkv, G, 1));
+    part = std::max(part, seedk::attn_tc_part_bound(G, 1));
   if (seedk::attn_tc_supported(cfg->head_dim, G, cfg->kmax + 1))
-    part = std::max(part, seedk::attn_tc_part_bound(batch, cfg->hkv, G, cfg->kmax + 1));
+    part = std::max(part, seedk::attn_tc_part_bound(G, cfg->kmax + 1));
   return kSchedBytes + counters_bytes(cfg, batch) + round_up(part, kAlign);
 }
 
