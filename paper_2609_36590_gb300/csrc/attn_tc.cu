@@ -60,19 +60,22 @@ constexpr int kD = 128;
 constexpr int kN = 128;                      // tokens (columns) per tile
 constexpr int kPagesPerTile = kN / kPage;    // 8
 constexpr int kStagesTC = 3;
-constexpr int kThreadsTC = 384;   // warps 0-7 softmax, 8-9 idle, 10 TMA producer, 11 MMA
-constexpr int kWarpProducer = 10, kWarpMma = 11;
+constexpr int kThreadsTC = 384;   // warps 0-7 softmax, 8 idle, 9 V loads, 10 K loads, 11 MMA
+constexpr int kWarpLoadV = 9, kWarpProducer = 10, kWarpMma = 11;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kColO = 256;              // O accumulators: [256, 384) and [384, 512)
 constexpr float kRescale = 8.0f;
 constexpr float kLn2 = 0.69314718055994531f;
 constexpr unsigned kFull = 0xffffffffu;
 
+constexpr int kMetaRing = 2 * kStagesTC;      // tile descriptors in flight
+
 constexpr uint32_t kHalf = kN * 128;                   // 16 KiB: 128 rows x 128 B
 constexpr uint32_t kQBytes = 2 * kHalf;                // Q: two head-dim halves
-constexpr uint32_t kStageBytes = 4 * kHalf;            // K0 K1 V0 V1
-constexpr uint32_t kOffStages = kQBytes;
-constexpr uint32_t kOffCtrl = kOffStages + kStagesTC * kStageBytes;
+constexpr uint32_t kKV = 2 * kHalf;                    // one tile's K (or V): two halves
+constexpr uint32_t kOffK = kQBytes;                    // K ring
+constexpr uint32_t kOffV = kOffK + kStagesTC * kKV;    // V ring
+constexpr uint32_t kOffCtrl = kOffV + kStagesTC * kKV;
 
 constexpr uint32_t kIdescS = idesc_bf16_f32(128, kN, 0, 0);     // K-major A and B
 constexpr uint32_t kIdescPV = idesc_bf16_f32(128, kD, 0, 1);    // B (V) MN-major
@@ -87,18 +90,23 @@ struct TileMeta {
   int32_t cvalid;      // cache rows that exist (L, or L + n_q for verify)
   int32_t lim0;        // query j sees cache positions <= lim0 + j
   int32_t slot;        // partial record of this piece, or -1: the whole pair
-  int32_t pad[4];
+  int32_t dslot;       // page slot of the draft rows in this tile, or -1
+  int32_t pad[3];
+  int32_t pids[kPagesPerTile];   // cache page of each page slot, -1: none
 };
 
 struct Ctrl {
-  uint64_t kv_full[kStagesTC];
-  uint64_t kv_empty[kStagesTC];
+  uint64_t k_full[kStagesTC], k_empty[kStagesTC];   // K ring
+  uint64_t v_full[kStagesTC], v_empty[kStagesTC];   // V ring
   uint64_t q_full, q_empty;
+  uint64_t end_bar;                           // the MMA thread's drain at the end
+  uint64_t meta_full[kMetaRing], meta_empty[kMetaRing];   // K warp -> V warp
   uint64_t s_full[2], p_full[2], o_full[2];   // per tile parity
   uint64_t stats_bar[4], orel_bar[4];         // per TMEM lane quarter
   uint32_t tmem_base;
   volatile int32_t abort_flag;
-  TileMeta meta[kStagesTC];
+  int32_t end_tile;                           // first tile index past the CTA's work
+  TileMeta meta[kMetaRing];
   float xm[4][32], xl[4][32];                 // row statistics handed to the epilogue owner
 };
 
@@ -118,6 +126,12 @@ __device__ __noinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, Ctrl*
   c->abort_flag = 1;
   raise_err(err, SEED_DEVERR_TIMEOUT);
   return false;
+}
+
+// Bounded wait by a whole warp: the lanes agree on the outcome, so that an
+// abort racing with the barrier's completion cannot split the warp.
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, Ctrl* c, int32_t* err) {
+  return __all_sync(0xffffffffu, wait_or_abort(bar, parity, c, err));
 }
 
 // ------------------------------------------------------------- sequences
@@ -496,14 +510,21 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
   const uint32_t sbase = smem_u32(smem);
 
   if (tid == 0) {
+    // one arrival per lane quarter that can hold query rows in this launch
+    const int nqa = min(4, (p.G * p.W1 + 31) / 32);
     for (int s = 0; s < kStagesTC; ++s) {
-      mbar_init(&ctrl->kv_full[s], 1);
-      mbar_init(&ctrl->kv_empty[s], 1);
+      mbar_init(&ctrl->k_full[s], 1);
+      mbar_init(&ctrl->k_empty[s], 1);
+      mbar_init(&ctrl->v_full[s], 1);
+      mbar_init(&ctrl->v_empty[s], 1);
     }
     mbar_init(&ctrl->q_full, 1);
     mbar_init(&ctrl->q_empty, 1);
-    // one arrival per lane quarter that can hold query rows in this launch
-    const int nqa = min(4, (p.G * p.W1 + 31) / 32);
+    mbar_init(&ctrl->end_bar, 1);
+    for (int i = 0; i < kMetaRing; ++i) {
+      mbar_init(&ctrl->meta_full[i], 1);
+      mbar_init(&ctrl->meta_empty[i], 1);
+    }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&ctrl->s_full[i], 1);
       mbar_init(&ctrl->p_full[i], nqa);
@@ -514,6 +535,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
       mbar_init(&ctrl->orel_bar[i], 1);
     }
     ctrl->abort_flag = 0;
+    ctrl->end_tile = 1 << 30;
     fence_mbar_init();
   }
   if (warp == kWarpMma) {
@@ -550,34 +572,53 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
     SeqWin win;
     int b = p.B, g = 0, t0 = 0;
     if (x < x1) locate(p, x, lane, win, b, g, t0);
-    int it = 0, uo = 0;
+    // K tiles in range order, each into the K ring as soon as a slot is free
+    // (a slot frees when S of its tile is done).  Each tile's descriptor goes
+    // to the descriptor ring, from which the V warp issues the tile's V.
+    int tk = 0, uo = 0;
     bool ok = true;
+    // page ids of tiles t and t + 1 of the piece (lanes 0-7, one page each),
+    // loaded ahead so that their latency overlaps the copies
+    int pid_a = -1, pid_b = -1;
+    SeqT sq{};
+    int t1 = 0;
+    auto load_pid = [&](int tt) -> int {
+      const int vp = tt * kPagesPerTile + (lane & 7);
+      return (lane < kPagesPerTile && tt < t1 && vp < sq.ncp)
+                 ? __ldg(p.page_table + (size_t)b * p.max_pages + vp)
+                 : -1;
+    };
     while (ok && x < x1 && b < p.B) {
       // one piece: tiles [t0, t1) of pair (b, g)
-      const SeqT sq = win_get(win, b);
-      const int t1 = (int)min((long long)sq.tiles, t0 + (x1 - x));
+      sq = win_get(win, b);
+      t1 = (int)min((long long)sq.tiles, t0 + (x1 - x));
       const int slot = (t0 == 0 && t1 == sq.tiles) ? -1 : 2 * (int)blockIdx.x + (uo > 0 ? 1 : 0);
-      for (int t = t0; t < t1 && ok; ++t, ++it) {
-        const int s = it % kStagesTC;
-        // page ids of this tile, one lane per page
-        const int vp = t * kPagesPerTile + (lane & 7);
-        int pid = -1;
-        if (lane < kPagesPerTile && vp < sq.ncp) {
-          pid = p.page_table[(size_t)b * p.max_pages + vp];
-          if (pid < 0 || pid >= p.num_pages) {
-            raise_err(p.err, SEED_DEVERR_PAGE);
-            pid = -1;
-          }
-        }
-        if (it >= kStagesTC)
-          ok = wait_or_abort(&ctrl->kv_empty[s], ((it / kStagesTC) - 1) & 1, ctrl, p.err);
-        if (ok && t == t0 && uo > 0) ok = wait_or_abort(&ctrl->q_empty, (uo - 1) & 1, ctrl, p.err);
+      pid_a = load_pid(t0);
+      pid_b = load_pid(t0 + 1);
+      for (int t = t0; t < t1; ++t, ++tk) {
+        const int s = tk % kStagesTC, mi = tk % kMetaRing;
+        int pid = pid_a;
+        pid_a = pid_b;
+        pid_b = load_pid(t + 2);
+        if (tk >= kStagesTC)
+          ok = warp_wait(&ctrl->k_empty[s], ((tk / kStagesTC) - 1) & 1, ctrl, p.err);
+        if (ok && tk >= kMetaRing)
+          ok = warp_wait(&ctrl->meta_empty[mi], ((tk / kMetaRing) - 1) & 1, ctrl, p.err);
+        if (ok && t == t0 && uo > 0) ok = warp_wait(&ctrl->q_empty, (uo - 1) & 1, ctrl, p.err);
         if (!ok) break;
-        int pids[kPagesPerTile];
-#pragma unroll
-        for (int pp = 0; pp < kPagesPerTile; ++pp) pids[pp] = __shfl_sync(kFull, pid, pp);
+        if (lane < kPagesPerTile && t * kPagesPerTile + lane < sq.ncp &&
+            (pid < 0 || pid >= p.num_pages)) {
+          raise_err(p.err, SEED_DEVERR_PAGE);
+          pid = -1;
+        }
+        // lane pp < 8 owns page slot pp of the tile
+        const int dslot = sq.nd > 0 ? sq.ncp - t * kPagesPerTile : -1;
+        const bool has = lane < kPagesPerTile && (pid >= 0 || lane == dslot);
+        const uint32_t loads = __ballot_sync(kFull, has);
+        TileMeta& m = ctrl->meta[mi];
+        if (lane < kPagesPerTile) m.pids[lane] = pid;
+        __syncwarp();
         if (lane == 0) {
-          TileMeta& m = ctrl->meta[s];
           m.unit = uo;
           m.b = b;
           m.g = g;
@@ -590,34 +631,26 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
           m.cvalid = sq.cvalid;
           m.lim0 = sq.lim0;
           m.slot = slot;
+          m.dslot = dslot;
+          mbar_arrive(&ctrl->meta_full[mi]);
           if (t == t0) {
             mbar_arrive_expect_tx(&ctrl->q_full, 2u * 128u * (uint32_t)Rmax);
             tma_load_4d(smem, &tm_q, 0, g * p.G, 0, b, &ctrl->q_full);
             tma_load_4d(smem + kHalf, &tm_q, 64, g * p.G, 0, b, &ctrl->q_full);
           }
-          const int dslot = sq.nd > 0 ? sq.ncp - t * kPagesPerTile : -1;   // draft page slot
-          uint32_t bytes = 0;
-#pragma unroll
-          for (int pp = 0; pp < kPagesPerTile; ++pp)
-            if (pids[pp] >= 0 || pp == dslot) bytes += 4u * 2048u;
-          mbar_arrive_expect_tx(&ctrl->kv_full[s], bytes);
-          uint8_t* st = smem + kOffStages + (size_t)s * kStageBytes;
-#pragma unroll 1
-          for (int pp = 0; pp < kPagesPerTile; ++pp) {
-            const bool is_draft = pids[pp] < 0 && pp == dslot;
-            if (pids[pp] < 0 && !is_draft) continue;
-            const CUtensorMap* mk = is_draft ? &tm_dk : &tm_k;
-            const CUtensorMap* mv = is_draft ? &tm_dv : &tm_v;
-            const int w = is_draft ? b : pids[pp];
-            const uint32_t off = pp * 2048u;
-            tma_load_4d(st + 0 * kHalf + off, mk, 0, 0, g, w, &ctrl->kv_full[s]);
-            tma_load_4d(st + 1 * kHalf + off, mk, 64, 0, g, w, &ctrl->kv_full[s]);
-            tma_load_4d(st + 2 * kHalf + off, mv, 0, 0, g, w, &ctrl->kv_full[s]);
-            tma_load_4d(st + 3 * kHalf + off, mv, 64, 0, g, w, &ctrl->kv_full[s]);
-          }
+          mbar_arrive_expect_tx(&ctrl->k_full[s], (uint32_t)__popc(loads) * 2u * 2048u);
         }
         __syncwarp();
+        if (has) {
+          const bool is_draft = pid < 0;
+          uint8_t* kb = smem + kOffK + (size_t)s * kKV + lane * 2048u;
+          const CUtensorMap* mk = is_draft ? &tm_dk : &tm_k;
+          const int w = is_draft ? b : pid;
+          tma_load_4d(kb, mk, 0, 0, g, w, &ctrl->k_full[s]);
+          tma_load_4d(kb + kHalf, mk, 64, 0, g, w, &ctrl->k_full[s]);
+        }
       }
+      if (!ok) break;
       ++uo;
       x += t1 - t0;
       if (x >= x1) break;
@@ -628,15 +661,52 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
         next_seq(p, lane, win, b);
       }
     }
-    // end markers: one for each softmax parity (the MMA thread stops at the first)
-    for (int e = 0; e < 2 && ok; ++e, ++it) {
-      const int s = it % kStagesTC;
-      if (it >= kStagesTC) ok = wait_or_abort(&ctrl->kv_empty[s], ((it / kStagesTC) - 1) & 1, ctrl, p.err);
+    // end markers: one for each softmax parity (the MMA thread stops at the
+    // first, the V warp too)
+    for (int e = 0; e < 2 && ok; ++e, ++tk) {
+      const int s = tk % kStagesTC, mi = tk % kMetaRing;
+      if (tk >= kStagesTC)
+        ok = warp_wait(&ctrl->k_empty[s], ((tk / kStagesTC) - 1) & 1, ctrl, p.err);
+      if (ok && tk >= kMetaRing)
+        ok = warp_wait(&ctrl->meta_empty[mi], ((tk / kMetaRing) - 1) & 1, ctrl, p.err);
       if (ok && lane == 0) {
-        ctrl->meta[s].unit = -1;
-        mbar_arrive(&ctrl->kv_full[s]);
+        ctrl->meta[mi].unit = -1;
+        mbar_arrive(&ctrl->meta_full[mi]);
+        mbar_arrive(&ctrl->k_full[s]);
       }
     }
+    __syncwarp();
+  } else if (warp == kWarpLoadV) {
+    // ---------------------------------------------------------- V loads
+    // V(t) into the V ring once tile t's descriptor is out and PV(t - 3)
+    // has freed the slot
+    for (int tv = 0;; ++tv) {
+      const int s = tv % kStagesTC, mi = tv % kMetaRing;
+      if (!warp_wait(&ctrl->meta_full[mi], (tv / kMetaRing) & 1, ctrl, p.err)) break;
+      const TileMeta& m = ctrl->meta[mi];
+      if (m.unit < 0) break;
+      const int pid = lane < kPagesPerTile ? m.pids[lane] : -1;
+      const int mb = m.b, mg = m.g, dslot = m.dslot;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctrl->meta_empty[mi]);
+      if (tv >= kStagesTC &&
+          !warp_wait(&ctrl->v_empty[s], ((tv / kStagesTC) - 1) & 1, ctrl, p.err))
+        break;
+      const bool has = lane < kPagesPerTile && (pid >= 0 || lane == dslot);
+      const uint32_t loads = __ballot_sync(kFull, has);
+      if (lane == 0)
+        mbar_arrive_expect_tx(&ctrl->v_full[s], (uint32_t)__popc(loads) * 2u * 2048u);
+      __syncwarp();
+      if (has) {
+        const bool is_draft = pid < 0;
+        uint8_t* vb = smem + kOffV + (size_t)s * kKV + lane * 2048u;
+        const CUtensorMap* mv = is_draft ? &tm_dv : &tm_v;
+        const int w = is_draft ? mb : pid;
+        tma_load_4d(vb, mv, 0, 0, mg, w, &ctrl->v_full[s]);
+        tma_load_4d(vb + kHalf, mv, 64, 0, mg, w, &ctrl->v_full[s]);
+      }
+    }
+    __syncwarp();
   } else if (warp == kWarpMma) {
     // ---------------------------------------------------------- MMA issuer
     // An event loop over two streams: S(ts) = Q K^T of the next loaded tile
@@ -652,20 +722,29 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
         bool did = false;
         if (ts < t_end && ts <= tp + 1) {
           const int s = ts % kStagesTC;
-          if (mbar_test(&ctrl->kv_full[s], (ts / kStagesTC) & 1)) {
-            const int unit = ctrl->meta[s].unit;
+          const TileMeta& mt = ctrl->meta[ts % kMetaRing];
+          if (mbar_test(&ctrl->k_full[s], (ts / kStagesTC) & 1)) {
+            const int unit = mt.unit;
             if (unit < 0) {
+              // no more tiles: wake both softmax groups through their S
+              // barriers (their next tiles, ts and ts + 1, never get an S),
+              // once every earlier S has completed and signalled
               t_end = ts;
+              mma_commit(&ctrl->end_bar);
+              if (!wait_or_abort(&ctrl->end_bar, 0, ctrl, p.err)) break;
+              ctrl->end_tile = ts;
+              mbar_arrive(&ctrl->s_full[ts & 1]);
+              mbar_arrive(&ctrl->s_full[(ts + 1) & 1]);
               did = true;
             } else {
-              const int k = ctrl->meta[s].k;
+              const int k = mt.k;
               const bool q_ok = (k != 0) || mbar_test(&ctrl->q_full, uo & 1);
               if (q_ok) {
                 if (k == 0) ++uo;
                 k_of[s] = k;
                 tc_fence_after();
                 const uint32_t d = tmem + (uint32_t)(ts & 1) * kN;
-                const uint32_t kb = sbase + kOffStages + (uint32_t)s * kStageBytes;
+                const uint32_t kb = sbase + kOffK + (uint32_t)s * kKV;
 #pragma unroll 1
                 for (int kk = 0; kk < kD / 16; ++kk) {
                   const uint32_t h = kk >> 2, off = (kk & 3) * 32;
@@ -674,19 +753,21 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
                   mma_ss(d, a, b, kIdescS, kk > 0);
                 }
                 mma_commit(&ctrl->s_full[ts & 1]);
-                if (ctrl->meta[s].k == ctrl->meta[s].ntu - 1) mma_commit(&ctrl->q_empty);
+                mma_commit(&ctrl->k_empty[s]);
+                if (mt.k == mt.ntu - 1) mma_commit(&ctrl->q_empty);
                 ++ts;
                 did = true;
               }
             }
           }
         }
-        if (tp < ts && mbar_test(&ctrl->p_full[tp & 1], (tp >> 1) & 1)) {
+        if (tp < ts && mbar_test(&ctrl->p_full[tp & 1], (tp >> 1) & 1) &&
+            mbar_test(&ctrl->v_full[tp % kStagesTC], (tp / kStagesTC) & 1)) {
           tc_fence_after();
           const int sp = tp % kStagesTC;
           const uint32_t pcol = tmem + (uint32_t)(tp & 1) * kN;
           const uint32_t ocol = tmem + kColO + (uint32_t)(tp & 1) * kD;
-          const uint32_t vb = sbase + kOffStages + (uint32_t)sp * kStageBytes + 2 * kHalf;
+          const uint32_t vb = sbase + kOffV + (uint32_t)sp * kKV;
           const bool first = k_of[sp] < 2;
           // tokens [16kk, 16kk+16): P_hi at packed column 32*(kk/2) + 8*(kk%2),
           // P_lo 16 columns further
@@ -698,7 +779,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
             mma_ts(ocol, a + 16, b, kIdescPV, 1);
           }
           mma_commit(&ctrl->o_full[tp & 1]);
-          mma_commit(&ctrl->kv_empty[sp]);
+          mma_commit(&ctrl->v_empty[sp]);
           ++tp;
           did = true;
         }
@@ -732,12 +813,15 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
     float m_used = -INFINITY, l = 0.f;
     int xcnt = 0;
     bool pend_rel = false;
-    for (int t = par, own = 0; !ctrl->abort_flag; t += 2, ++own) {
+    // (every wait below gives up once another role has aborted; the lanes
+    // agree on each outcome, so the loop is left by the whole warp at once)
+    for (int t = par, own = 0;; t += 2, ++own) {
       const int s = t % kStagesTC;
-      if (!wait_or_abort(&ctrl->kv_full[s], (t / kStagesTC) & 1, ctrl, p.err)) break;
-      const TileMeta m = ctrl->meta[s];
-      if (m.unit < 0) break;
-      if (!wait_or_abort(&ctrl->s_full[par], own & 1, ctrl, p.err)) break;
+      // S(t) done implies K(t) landed and tile t's descriptor is written; the
+      // MMA thread also completes this phase, without an S, at the end
+      if (!warp_wait(&ctrl->s_full[par], own & 1, ctrl, p.err)) break;
+      if (t >= *reinterpret_cast<volatile int32_t*>(&ctrl->end_tile)) break;
+      const TileMeta m = ctrl->meta[t % kMetaRing];
       tc_fence_after();
       const bool first_own = m.k < 2;
       if (first_own) {
@@ -772,7 +856,9 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
       // V rows of columns nobody may see are zeroed, so that a probability of
       // 0 never meets a stale or NaN-poisoned row
       if (m.cvalid - m.tile * kN < kN || cm.dcol < kN) {
-        uint8_t* vb = smem + kOffStages + (size_t)s * kStageBytes + 2 * kHalf;
+        // (after V has landed, or the copy engine would overwrite the zeros)
+        if (!warp_wait(&ctrl->v_full[s], (t / kStagesTC) & 1, ctrl, p.err)) break;
+        uint8_t* vb = smem + kOffV + (size_t)s * kKV;
         bool wrote = false;
 #pragma unroll 1
         for (int col = q4 * 32 + lane; col < kN; col += 32 * nqa) {
@@ -787,16 +873,19 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
         }
         if (wrote) fence_proxy_async_smem();
       }
-      // this group's previous PV must be done before its O is rescaled
-      if (own > 0 && !wait_or_abort(&ctrl->o_full[par], (own - 1) & 1, ctrl, p.err)) break;
+      // this group's previous PV must be done before its O is rescaled (the
+      // rescale is rare: only when the running maximum jumps by > 2^8)
+      const bool do_resc = warp_active && __any_sync(kFull, resc);
+      if (own > 0 && do_resc && !warp_wait(&ctrl->o_full[par], (own - 1) & 1, ctrl, p.err))
+        break;
       // the first tile of a unit overwrites O: the other group's epilogue of
       // the previous unit must have read it
       if (first_own && pend_rel) {
-        if (!wait_or_abort(&ctrl->orel_bar[q4], (xcnt - 1) & 1, ctrl, p.err)) break;
+        if (!warp_wait(&ctrl->orel_bar[q4], (xcnt - 1) & 1, ctrl, p.err)) break;
         pend_rel = false;
       }
       tc_fence_after();
-      if (warp_active && __any_sync(kFull, resc)) {
+      if (do_resc) {
         const float f = resc ? fo : 1.f;
 #pragma unroll 1
         for (int c = 0; c < kD / 32; ++c) {
@@ -815,7 +904,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
 
       if (m.k + 2 >= m.ntu) {
         // ------------------------------------------------ this group's last tile of the unit
-        if (!wait_or_abort(&ctrl->o_full[par], own & 1, ctrl, p.err)) break;
+        if (!warp_wait(&ctrl->o_full[par], own & 1, ctrl, p.err)) break;
         tc_fence_after();
         if (m.k != m.ntu - 1) {
           // the other group owns the epilogue: hand over this row's statistics
@@ -830,7 +919,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
           // ---------------------------------------------- epilogue (owner)
           float mo = -INFINITY, lo = 0.f;
           if (m.ntu >= 2) {
-            if (!wait_or_abort(&ctrl->stats_bar[q4], xcnt & 1, ctrl, p.err)) break;
+            if (!warp_wait(&ctrl->stats_bar[q4], xcnt & 1, ctrl, p.err)) break;
             tc_fence_after();
             mo = ctrl->xm[q4][lane];
             lo = ctrl->xl[q4][lane];
