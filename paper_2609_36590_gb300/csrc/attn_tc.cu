@@ -99,7 +99,6 @@ struct Ctrl {
   uint64_t k_full[kStagesTC], k_empty[kStagesTC];   // K ring
   uint64_t v_full[kStagesTC], v_empty[kStagesTC];   // V ring
   uint64_t q_full, q_empty;
-  uint64_t end_bar;                           // the MMA thread's drain at the end
   uint64_t meta_full[kMetaRing], meta_empty[kMetaRing];   // K warp -> V warp
   uint64_t s_full[2], p_full[2], o_full[2];   // per tile parity
   uint64_t stats_bar[4], orel_bar[4];         // per TMEM lane quarter
@@ -168,10 +167,13 @@ __device__ __forceinline__ SeqT seq_of(const AttnTcParams& p, int b) {
 }
 
 // ------------------------------------------------------------- partition
-// Tiles of the launch: T = hkv * sum_b tiles(b).  CTA c of N takes the tiles
-// [start(c), start(c+1)) with start(c) = floor(c T / N) when T >= N (every
-// range non-empty), else start(c) = min(c, T) (one tile each for the first T
-// CTAs), so that the CTAs holding one pair are always consecutive.
+// The launch's work as a line of cost units: pair (b, g) with tiles(b) > 0
+// takes kPairCost units for its fixed cost (descriptor and Q load, first-tile
+// latency, epilogue), then one unit per tile; pairs in (b, g) order.  CTA c of
+// N owns the units [start(c), start(c+1)) with start(c) = floor(c T / N) when
+// T >= N, else min(c, T), and so the tiles whose units fall there: a
+// contiguous run of pieces, and the CTAs holding one pair are consecutive.
+constexpr int kPairCost = 2;
 __device__ __forceinline__ long long range_start(long long T, int c, int N) {
   return T >= N ? T * c / N : min((long long)c, T);
 }
@@ -181,12 +183,17 @@ __device__ __forceinline__ int cta_of(long long x, long long T, int N) {
   return T >= N ? (int)(((x + 1) * N - 1) / T) : (int)x;
 }
 
+// Cost units of all pairs of sequence b.
+__device__ __forceinline__ long long seq_cost(const AttnTcParams& p, int tiles) {
+  return tiles > 0 ? (long long)p.hkv * (tiles + kPairCost) : 0;
+}
+
 // Warp-cooperative: T.
-__device__ __noinline__ long long total_tiles(const AttnTcParams& p, int lane) {
+__device__ __noinline__ long long total_cost(const AttnTcParams& p, int lane) {
   long long tot = 0;
-  for (int b = lane; b < p.B; b += 32) tot += seq_of(p, b).tiles;
+  for (int b = lane; b < p.B; b += 32) tot += seq_cost(p, seq_of(p, b).tiles);
   for (int o = 16; o; o >>= 1) tot += __shfl_xor_sync(kFull, tot, o);
-  return tot * p.hkv;
+  return tot;
 }
 
 // A window of 32 sequences [wb, wb + 32); lane i holds sequence wb + i.
@@ -212,14 +219,15 @@ __device__ __forceinline__ SeqT win_get(const SeqWin& w, int b) {
   return s;
 }
 
-// Warp-cooperative: the (sequence b, KV head g, tile t) of tile x < T, with
-// the window that holds b.
+// Warp-cooperative: the pair (sequence b, KV head g) whose units hold unit
+// x < T, the first unit pc of that pair, and the first tile t at or after x
+// (0 when x falls in the pair's fixed-cost units); with the window that holds b.
 __device__ __noinline__ void locate(const AttnTcParams& p, long long x, int lane, SeqWin& w,
-                                    int& b, int& g, int& t) {
+                                    int& b, int& g, int& t, long long& pc) {
   long long base = 0;
   for (w.wb = 0; w.wb < p.B; w.wb += 32) {
     w.mine = seq_or_empty(p, w.wb + lane);
-    const long long a = (long long)p.hkv * w.mine.tiles;
+    const long long a = seq_cost(p, w.mine.tiles);
     long long inc = a;
     for (int o = 1; o < 32; o <<= 1) {
       const long long v = __shfl_up_sync(kFull, inc, o);
@@ -229,17 +237,19 @@ __device__ __noinline__ void locate(const AttnTcParams& p, long long x, int lane
     if (x < base + tot) {
       const unsigned m = __ballot_sync(kFull, base + inc - a <= x && x < base + inc);
       const int src = __ffs(m) - 1;
-      const long long r = x - base - __shfl_sync(kFull, inc - a, src);
-      const int tiles = __shfl_sync(kFull, w.mine.tiles, src);
+      const long long sb = base + __shfl_sync(kFull, inc - a, src);
+      const int per = __shfl_sync(kFull, w.mine.tiles, src) + kPairCost;
       b = w.wb + src;
-      g = (int)(r / tiles);
-      t = (int)(r - (long long)g * tiles);
+      g = (int)((x - sb) / per);
+      pc = sb + (long long)g * per;
+      t = (int)max(0LL, x - pc - kPairCost);
       return;
     }
     base += tot;
   }
   b = p.B;
   g = t = 0;
+  pc = 0;
 }
 
 // Warp-cooperative: the next sequence after b with at least one tile (p.B if
@@ -389,22 +399,24 @@ __device__ __noinline__ void unit_epilogue(const AttnTcParams& p, int b, int g, 
 // Merge of the pieces of pair (b, g) = (blockIdx.x / hkv, blockIdx.x % hkv)
 // when the pair's tiles span several CTAs of the attention kernel: the
 // pieces' records are combined with weights 2^(lse_i - M) / sum, in range
-// order.  Pairs that one CTA finished alone return at once.  Loads are
-// issued kMergeBatch pieces at a time so that their latencies overlap.
+// order.  One warp per query row (rows 8 * blockIdx.y + warp), one lane per 4
+// head dims; each lane reads every piece's log2-sum-exp and values in one
+// online pass, kMergeBatch pieces at a time.  Pairs that one CTA finished
+// alone return at once.
 constexpr int kMergeThreads = 256;
+constexpr int kMergeRows = kMergeThreads / 32;
 constexpr int kMergeBatch = 8;
 
 __global__ void __launch_bounds__(kMergeThreads) attn_merge_kernel(const AttnTcParams p) {
-  __shared__ long long red[2][kMergeThreads / 32];
-  __shared__ float s_m[128], s_inv[128];
+  __shared__ long long red[2][kMergeRows];
   const int pair = blockIdx.x;
   const int b = pair / p.hkv, g = pair - b * p.hkv;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   long long tot = 0, pre = 0;
   for (int i = tid; i < p.B; i += kMergeThreads) {
-    const int t = seq_of(p, i).tiles;
-    tot += t;
-    if (i < b) pre += t;
+    const long long c = seq_cost(p, seq_of(p, i).tiles);
+    tot += c;
+    if (i < b) pre += c;
   }
   for (int o = 16; o; o >>= 1) {
     tot += __shfl_xor_sync(kFull, tot, o);
@@ -417,80 +429,64 @@ __global__ void __launch_bounds__(kMergeThreads) attn_merge_kernel(const AttnTcP
   __syncthreads();
   tot = pre = 0;
 #pragma unroll
-  for (int w = 0; w < kMergeThreads / 32; ++w) {
+  for (int w = 0; w < kMergeRows; ++w) {
     tot += red[0][w];
     pre += red[1][w];
   }
   const SeqT sq = seq_of(p, b);
-  if (sq.tiles == 0) return;
-  const long long T = tot * p.hkv;
-  const long long P0 = pre * p.hkv + (long long)g * sq.tiles, P1 = P0 + sq.tiles;
-  const int c_lo = cta_of(P0, T, p.nctas), c_hi = cta_of(P1 - 1, T, p.nctas);
+  const int r = blockIdx.y * kMergeRows + warp;   // query row j * G + head
+  if (sq.tiles == 0 || r >= sq.nq * p.G) return;
+  const long long T = tot;
+  const long long pc = pre + (long long)g * (sq.tiles + kPairCost);   // the pair's first unit
+  const long long u0 = pc + kPairCost, u1 = u0 + sq.tiles - 1;         // its first and last tile
+  const int c_lo = cta_of(u0, T, p.nctas), c_hi = cta_of(u1, T, p.nctas);
   if (c_lo == c_hi) return;
   const int nseg = c_hi - c_lo + 1;
-  // the piece of CTA c_lo is its first piece if its range starts with it
-  const int slot_lo = 2 * c_lo + (range_start(T, c_lo, p.nctas) == P0 ? 0 : 1);
+  // the piece of CTA c_lo is its first piece unless the range of c_lo starts
+  // before the pair (then it holds the previous pair's last tile, unit pc - 1)
+  const int slot_lo = 2 * c_lo + (range_start(T, c_lo, p.nctas) >= pc ? 0 : 1);
   const int Rmax = p.G * p.W1;
   const size_t REC = (size_t)Rmax * (kD + 1);
-  const int R = sq.nq * p.G;
-  const float* lse_base = p.part + (size_t)kD * Rmax;    // + slot * REC + row
-  // row statistics: one online pass over the pieces' log2-sum-exps
-  for (int r = tid; r < R; r += kMergeThreads) {
-    float M = -INFINITY, S = 0.f;
-    for (int i0 = 0; i0 < nseg; i0 += kMergeBatch) {
-      float li[kMergeBatch];
+  float M = -INFINITY, S = 0.f;
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int i0 = 0; i0 < nseg; i0 += kMergeBatch) {
+    float li[kMergeBatch];
+    float4 x[kMergeBatch];
 #pragma unroll
-      for (int u = 0; u < kMergeBatch; ++u) {
-        const int i = min(i0 + u, nseg - 1);
-        const int slot = i == 0 ? slot_lo : 2 * (c_lo + i);
-        li[u] = (i0 + u < nseg) ? __ldcg(lse_base + slot * REC + r) : -INFINITY;
-      }
-#pragma unroll
-      for (int u = 0; u < kMergeBatch; ++u) {
-        if (li[u] == -INFINITY) continue;
-        if (li[u] > M) {
-          S = S * ex2_approx(M - li[u]) + 1.f;
-          M = li[u];
-        } else {
-          S += ex2_approx(li[u] - M);
-        }
-      }
+    for (int u = 0; u < kMergeBatch; ++u) {
+      const int i = min(i0 + u, nseg - 1);
+      const float* rc = p.part + (size_t)(i == 0 ? slot_lo : 2 * (c_lo + i)) * REC;
+      li[u] = (i0 + u < nseg) ? __ldcg(rc + (size_t)kD * Rmax + r) : -INFINITY;
+      x[u] = __ldcg(reinterpret_cast<const float4*>(rc + (size_t)r * kD) + lane);
     }
-    s_m[r] = M;
-    s_inv[r] = 1.f / S;
-    const int j = r / p.G;
-    const size_t orow = ((size_t)b * p.W1 + j) * p.hq + g * p.G + (r - j * p.G);
-    if (p.lse != nullptr) p.lse[orow] = (M + log2f(S)) * kLn2;
-  }
-  __syncthreads();
-  for (int item = tid; item < R * (kD / 4); item += kMergeThreads) {
-    const int r = item / (kD / 4), c4 = item - r * (kD / 4);
-    const float M = s_m[r], inv = s_inv[r];
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int i0 = 0; i0 < nseg; i0 += kMergeBatch) {
-      float li[kMergeBatch];
-      float4 x[kMergeBatch];
 #pragma unroll
-      for (int u = 0; u < kMergeBatch; ++u) {
-        const int i = min(i0 + u, nseg - 1);
-        const int slot = i == 0 ? slot_lo : 2 * (c_lo + i);
-        const float* rc = p.part + slot * REC;
-        li[u] = (i0 + u < nseg) ? __ldcg(rc + (size_t)kD * Rmax + r) : -INFINITY;
-        x[u] = __ldcg(reinterpret_cast<const float4*>(rc + (size_t)r * kD) + c4);
+    for (int u = 0; u < kMergeBatch; ++u) {
+      if (li[u] == -INFINITY) continue;
+      float w = 1.f;
+      if (li[u] > M) {
+        const float f = ex2_approx(M - li[u]);   // 0 for the first piece
+        S *= f;
+        acc.x *= f;
+        acc.y *= f;
+        acc.z *= f;
+        acc.w *= f;
+        M = li[u];
+      } else {
+        w = ex2_approx(li[u] - M);
       }
-#pragma unroll
-      for (int u = 0; u < kMergeBatch; ++u) {
-        const float w = (li[u] == -INFINITY) ? 0.f : ex2_approx(li[u] - M) * inv;
-        acc.x = fmaf(w, x[u].x, acc.x);
-        acc.y = fmaf(w, x[u].y, acc.y);
-        acc.z = fmaf(w, x[u].z, acc.z);
-        acc.w = fmaf(w, x[u].w, acc.w);
-      }
+      S += w;
+      acc.x = fmaf(w, x[u].x, acc.x);
+      acc.y = fmaf(w, x[u].y, acc.y);
+      acc.z = fmaf(w, x[u].z, acc.z);
+      acc.w = fmaf(w, x[u].w, acc.w);
     }
-    const int j = r / p.G;
-    const size_t orow = ((size_t)b * p.W1 + j) * p.hq + g * p.G + (r - j * p.G);
-    reinterpret_cast<float4*>(p.out + orow * kD)[c4] = acc;
   }
+  const float inv = 1.f / S;
+  const int j = r / p.G;
+  const size_t orow = ((size_t)b * p.W1 + j) * p.hq + g * p.G + (r - j * p.G);
+  reinterpret_cast<float4*>(p.out + orow * kD)[lane] =
+      make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
+  if (lane == 0 && p.lse != nullptr) p.lse[orow] = (M + log2f(S)) * kLn2;
 }
 
 // No __launch_bounds__: with it ptxas budgets the 320-thread block like a
@@ -520,7 +516,6 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
     }
     mbar_init(&ctrl->q_full, 1);
     mbar_init(&ctrl->q_empty, 1);
-    mbar_init(&ctrl->end_bar, 1);
     for (int i = 0; i < kMetaRing; ++i) {
       mbar_init(&ctrl->meta_full[i], 1);
       mbar_init(&ctrl->meta_empty[i], 1);
@@ -565,13 +560,14 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
         if (bad) raise_err(p.err, bad);
       }
     }
-    // this CTA's range [x, x1) of the launch's tiles
-    const long long T = total_tiles(p, lane);
-    long long x = range_start(T, blockIdx.x, p.nctas);
+    // this CTA's units [x, x1)
+    const long long T = total_cost(p, lane);
+    const long long x = range_start(T, blockIdx.x, p.nctas);
     const long long x1 = range_start(T, blockIdx.x + 1, p.nctas);
     SeqWin win;
     int b = p.B, g = 0, t0 = 0;
-    if (x < x1) locate(p, x, lane, win, b, g, t0);
+    long long pc = 0;   // first unit of pair (b, g)
+    if (x < x1) locate(p, x, lane, win, b, g, t0, pc);
     // K tiles in range order, each into the K ring as soon as a slot is free
     // (a slot frees when S of its tile is done).  Each tile's descriptor goes
     // to the descriptor ring, from which the V warp issues the tile's V.
@@ -588,10 +584,11 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
                  ? __ldg(p.page_table + (size_t)b * p.max_pages + vp)
                  : -1;
     };
-    while (ok && x < x1 && b < p.B) {
-      // one piece: tiles [t0, t1) of pair (b, g)
+    while (ok && b < p.B) {
+      // one piece: tiles [t0, t1) of pair (b, g), those whose units lie below x1
       sq = win_get(win, b);
-      t1 = (int)min((long long)sq.tiles, t0 + (x1 - x));
+      t1 = (int)min((long long)sq.tiles, x1 - pc - kPairCost);
+      if (t1 <= t0) break;
       const int slot = (t0 == 0 && t1 == sq.tiles) ? -1 : 2 * (int)blockIdx.x + (uo > 0 ? 1 : 0);
       pid_a = load_pid(t0);
       pid_b = load_pid(t0 + 1);
@@ -652,9 +649,9 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
       }
       if (!ok) break;
       ++uo;
-      x += t1 - t0;
-      if (x >= x1) break;
+      if (t1 < sq.tiles) break;
       // the range goes on with the next pair
+      pc += sq.tiles + kPairCost;
       t0 = 0;
       if (++g == p.hkv) {
         g = 0;
@@ -726,15 +723,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
           if (mbar_test(&ctrl->k_full[s], (ts / kStagesTC) & 1)) {
             const int unit = mt.unit;
             if (unit < 0) {
-              // no more tiles: wake both softmax groups through their S
-              // barriers (their next tiles, ts and ts + 1, never get an S),
-              // once every earlier S has completed and signalled
-              t_end = ts;
-              mma_commit(&ctrl->end_bar);
-              if (!wait_or_abort(&ctrl->end_bar, 0, ctrl, p.err)) break;
-              ctrl->end_tile = ts;
-              mbar_arrive(&ctrl->s_full[ts & 1]);
-              mbar_arrive(&ctrl->s_full[(ts + 1) & 1]);
+              t_end = ts;   // no more tiles
               did = true;
             } else {
               const int k = mt.k;
@@ -791,6 +780,15 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
           ctrl->abort_flag = 1;
           raise_err(p.err, SEED_DEVERR_TIMEOUT);
         }
+      }
+      // Wake both softmax groups through their S barriers: their next tiles,
+      // t_end and t_end + 1, never get an S.  Only now: every PV has been
+      // issued, so each group has consumed all of its S phases and waits (or
+      // will wait) for exactly the phase these arrivals complete.
+      if (!ctrl->abort_flag) {
+        ctrl->end_tile = t_end;
+        mbar_arrive(&ctrl->s_full[t_end & 1]);
+        mbar_arrive(&ctrl->s_full[(t_end + 1) & 1]);
       }
     }
     __syncwarp();
@@ -1034,7 +1032,8 @@ cudaError_t launch_attn_tc(const AttnTcParams& prm, const void* q, const void* k
   attn_tc_kernel<<<prm.nctas, kThreadsTC, kSmemTC, st>>>(tq, tk, tv, tdk, tdv, prm);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  attn_merge_kernel<<<prm.B * prm.hkv, kMergeThreads, 0, st>>>(prm);
+  const dim3 mgrid(prm.B * prm.hkv, (prm.G * prm.W1 + kMergeRows - 1) / kMergeRows);
+  attn_merge_kernel<<<mgrid, kMergeThreads, 0, st>>>(prm);
   return cudaGetLastError();
 }
 

@@ -272,3 +272,36 @@ def test_device_errors_are_flagged_not_fatal(S):
     c["err"].zero_()
     out_ok, _ = run_verify(S, c, kv)
     assert int(c["err"].item()) == 0 and np.isfinite(out_ok[0, :c["n_q"][0]]).all()
+
+
+def test_many_short_pieces_repeated(S):
+    """Many 1-3 tile sequences: every CTA's range holds several pieces, each
+    with its own epilogue, so the hand-offs between the kernel's roles run
+    hundreds of times per launch.  Repeated draft and verify launches raise no
+    device error and keep matching the oracle."""
+    case = (96, 32, 8, 128, 8, 300, True, 1.0)
+    c = make(S, 7, case)
+    kv_d = kv_for(S, c, c["lens"])
+    kv_v = kv_for(S, c, c["lens"] + c["n_q"])
+    outs = []
+    for rep in range(12):
+        outs.append(run_draft(S, c, kv_d) if rep % 2 == 0 else run_verify(S, c, kv_v))
+        assert int(c["err"].item()) == 0, f"launch {rep}: device error {int(c['err'].item())}"
+    for rep in range(2, 12):
+        assert np.array_equal(outs[rep][0], outs[rep - 2][0]), f"launch {rep} differs"
+    od, ld = outs[0]
+    ov, lv = outs[1]
+    for b in range(0, case[0], 5):
+        dl, L, n = int(c["draft_lens"][b]), int(c["lens"][b]), int(c["n_q"][b])
+        if dl:
+            o, l = OAT.draft_attention_seq(
+                f64(c["q_draft"][b]), f64(c["rows_k"][b, :L]), f64(c["rows_v"][b, :L]),
+                f64(c["draft_k"][b, :, :dl].transpose(1, 0, 2)),
+                f64(c["draft_v"][b, :, :dl].transpose(1, 0, 2)), c["scale"])
+            assert_close(od[b], o, f"draft o b={b}")
+            assert_close(ld[b], l, f"draft lse b={b}")
+        if n:
+            o, l = OAT.verify_attention_seq(f64(c["q_verify"][b, :n]), f64(c["rows_k"][b, :L + n]),
+                                            f64(c["rows_v"][b, :L + n]), L, c["scale"])
+            assert_close(ov[b, :n], o, f"verify o b={b}")
+            assert_close(lv[b, :n], l, f"verify lse b={b}")
