@@ -12,7 +12,7 @@ row read once per attention call, queries, outputs, appended rows) / device
 time of the round.  Inputs are resident in HBM; a round's working set
 (gigabytes of KV) is far larger than the 129 MB L2.
 
-    python bench.py [--workload 3] [--steps 10] [--warmup 3] [--impl seed|reference]
+    python bench.py [--workload 4] [--steps 10] [--warmup 3] [--impl seed|reference]
 """
 
 from __future__ import annotations
@@ -81,10 +81,10 @@ def round_bytes(wl, lens: np.ndarray, k_b: np.ndarray, n_layers: int) -> dict:
 # reported traffic is scaled to the timed launches by their algorithmic bytes,
 # and is null once the kernel's sources differ from the captured ones.
 NCU_TRAFFIC = {
-    (3, "verify"): {"kernel": "attn_tc_kernel", "sources": "62a452f18ef2669c",
-                    "dram_bytes": 166086656 + 10738432, "alg_bytes": 165939200},
-    (3, "draft"): {"kernel": "attn_tc_kernel", "sources": "62a452f18ef2669c",
-                   "dram_bytes": 165008384 + 10237696, "alg_bytes": 164096000},
+    (4, "verify"): {"kernel": "attn_tc_kernel", "sources": "25fbed04a547802d",
+                    "dram_bytes": 538046208 + 10442240, "alg_bytes": 537907712},
+    (4, "draft"): {"kernel": "attn_tc_kernel", "sources": "25fbed04a547802d",
+                   "dram_bytes": 537460480 + 10101760, "alg_bytes": 536986112},
 }
 
 KERNEL_SOURCES = {
@@ -502,7 +502,7 @@ def main():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
-    ap.add_argument("--workload", type=int, default=3, choices=[1, 2, 3, 4, 5])
+    ap.add_argument("--workload", type=int, default=4, choices=[1, 2, 3, 4, 5])
     ap.add_argument("--impl", default="seed", choices=["seed", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=12.0)
