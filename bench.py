@@ -404,6 +404,21 @@ def run_profile(args):
                              for i in range(args.reps)]}))
 
 
+def aggregate(rank_bytes: float, rank_seconds: float, world: int, device="cpu"):
+    """Whole-job throughput of N replicas: every rank processed `rank_bytes` in
+    `rank_seconds`; the job takes as long as its slowest rank.  Returns
+    (max seconds over ranks, GB/s of all ranks together).  With world > 1 the
+    process group must be initialised (NCCL on GPUs, gloo on CPU)."""
+    import torch
+
+    total_s = float(rank_seconds)
+    if world > 1:
+        t = torch.tensor([total_s], dtype=torch.float64, device=device)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        total_s = float(t.item())
+    return total_s, world * rank_bytes / total_s / 1e9
+
+
 def count_launches(wl, steps_per_round, n_layers):
     nd = len(wl.dec_layers)
     return sum(2 * nd * s + 2 * n_layers + 1 for s in steps_per_round)
@@ -554,12 +569,7 @@ def main():
     device = f"cuda:{local}"
     res = run_seed(args, rank, world, device)
 
-    total_s = res["total_ms"] / 1e3
-    if world > 1:
-        t = torch.tensor([total_s], device=device)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total_s = float(t.item())
-    value = world * res["total_bytes"] / total_s / 1e9
+    total_s, value = aggregate(res["total_bytes"], res["total_ms"] / 1e3, world, device)
     if rank == 0:
         cpu = oracle_sample(wl, args.cpu_budget) if world == 1 else None
         K = args.steps
