@@ -409,6 +409,8 @@ constexpr int kMergeBatch = 8;
 
 __global__ void __launch_bounds__(kMergeThreads) attn_merge_kernel(const AttnTcParams p) {
   __shared__ long long red[2][kMergeRows];
+  if (threadIdx.x == 0) pdl_trigger();
+  pdl_wait();
   const int pair = blockIdx.x;
   const int b = pair / p.hkv, g = pair - b * p.hkv;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -489,13 +491,43 @@ __global__ void __launch_bounds__(kMergeThreads) attn_merge_kernel(const AttnTcP
   if (lane == 0 && p.lse != nullptr) p.lse[orow] = (M + log2f(S)) * kLn2;
 }
 
+// Tensor maps of the paged cache for boxes of 1, 2, 4 and 8 consecutive pages
+// (64 head dims x 16 rows x 1 KV head x n pages): n pages whose ids follow one
+// another are one copy, and land as 16 n consecutive 128-byte rows, the
+// swizzled K-major layout the MMAs read.
+struct PageMaps {
+  CUtensorMap k[4];
+  CUtensorMap v[4];
+};
+
+// Warp-cooperative: the copy box that lane s < 8 issues for page slot s of a
+// tile.  Runs of slots holding consecutive page ids are cut greedily into
+// boxes of 8, 4, 2 and 1 pages; the result is the box size if slot s starts a
+// box, else 0.  A slot at offset o of a run of n slots starts a box of
+// 2^floor(log2(n - o)) pages exactly when n with the bits below that box size
+// cleared equals o.
+__device__ __forceinline__ int box_size(int pid, int lane) {
+  const int pid_next = __shfl_down_sync(kFull, pid, 1);
+  const uint32_t valid = __ballot_sync(kFull, lane < kPagesPerTile && pid >= 0) & 0xffu;
+  const uint32_t cont =
+      __ballot_sync(kFull, lane < kPagesPerTile - 1 && pid >= 0 && pid_next == pid + 1) & 0x7fu;
+  if (lane >= kPagesPerTile || !((valid >> lane) & 1u)) return 0;
+  const uint32_t starts = valid & ~(cont << 1) & 0xffu;
+  const int r = 31 - __clz((int)(starts & ((2u << lane) - 1u)));   // first slot of the run
+  const int n = lane + __ffs((int)~(cont >> lane)) - r;            // slots in the run
+  const int o = lane - r;
+  const int sz = 1 << (31 - __clz(n - o));
+  return (n & ~(2 * sz - 1)) == o ? sz : 0;
+}
+
+__device__ __forceinline__ int log2_box(int sz) { return sz >= 8 ? 3 : sz >= 4 ? 2 : sz >= 2 ? 1 : 0; }
+
 // No __launch_bounds__: with it ptxas budgets the 320-thread block like a
 // 384-thread one and spills in the per-tile loop; without it the kernel fits
 // in 168 registers with no spills (a launch that did not fit would fail with
 // an error, never run).
 __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
-                   const __grid_constant__ CUtensorMap tm_k,
-                   const __grid_constant__ CUtensorMap tm_v,
+                   const __grid_constant__ PageMaps pm,
                    const __grid_constant__ CUtensorMap tm_dk,
                    const __grid_constant__ CUtensorMap tm_dv, const AttnTcParams p) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -504,6 +536,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
   Ctrl* ctrl = reinterpret_cast<Ctrl*>(smem + kOffCtrl);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint32_t sbase = smem_u32(smem);
+  if (tid == 0) pdl_trigger();
 
   if (tid == 0) {
     // one arrival per lane quarter that can hold query rows in this launch
@@ -542,13 +575,17 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
   tc_fence_after();
   const uint32_t tmem = ctrl->tmem_base;
   const int Rmax = p.G * p.W1;
+  // everything above touched only this CTA's shared and tensor memory
+  pdl_wait();
 
   if (warp == kWarpProducer) {
     // ---------------------------------------------------------- producer
     if (lane == 0) {
       tma_prefetch_desc(&tm_q);
-      tma_prefetch_desc(&tm_k);
-      tma_prefetch_desc(&tm_v);
+      for (int i = 0; i < 4; ++i) {
+        tma_prefetch_desc(&pm.k[i]);
+        tma_prefetch_desc(&pm.v[i]);
+      }
       if (p.draft) {
         tma_prefetch_desc(&tm_dk);
         tma_prefetch_desc(&tm_dv);
@@ -612,6 +649,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
         const int dslot = sq.nd > 0 ? sq.ncp - t * kPagesPerTile : -1;
         const bool has = lane < kPagesPerTile && (pid >= 0 || lane == dslot);
         const uint32_t loads = __ballot_sync(kFull, has);
+        const int box = box_size(pid, lane);
         TileMeta& m = ctrl->meta[mi];
         if (lane < kPagesPerTile) m.pids[lane] = pid;
         __syncwarp();
@@ -638,11 +676,11 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
           mbar_arrive_expect_tx(&ctrl->k_full[s], (uint32_t)__popc(loads) * 2u * 2048u);
         }
         __syncwarp();
-        if (has) {
-          const bool is_draft = pid < 0;
+        if (box > 0 || (has && pid < 0)) {
+          // a box of `box` pages from this slot on, or the draft rows' page
           uint8_t* kb = smem + kOffK + (size_t)s * kKV + lane * 2048u;
-          const CUtensorMap* mk = is_draft ? &tm_dk : &tm_k;
-          const int w = is_draft ? b : pid;
+          const CUtensorMap* mk = box > 0 ? &pm.k[log2_box(box)] : &tm_dk;
+          const int w = box > 0 ? pid : b;
           tma_load_4d(kb, mk, 0, 0, g, w, &ctrl->k_full[s]);
           tma_load_4d(kb + kHalf, mk, 64, 0, g, w, &ctrl->k_full[s]);
         }
@@ -694,11 +732,11 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
       if (lane == 0)
         mbar_arrive_expect_tx(&ctrl->v_full[s], (uint32_t)__popc(loads) * 2u * 2048u);
       __syncwarp();
-      if (has) {
-        const bool is_draft = pid < 0;
+      const int box = box_size(pid, lane);
+      if (box > 0 || (has && pid < 0)) {
         uint8_t* vb = smem + kOffV + (size_t)s * kKV + lane * 2048u;
-        const CUtensorMap* mv = is_draft ? &tm_dv : &tm_v;
-        const int w = is_draft ? mb : pid;
+        const CUtensorMap* mv = box > 0 ? &pm.v[log2_box(box)] : &tm_dv;
+        const int w = box > 0 ? pid : mb;
         tma_load_4d(vb, mv, 0, 0, mg, w, &ctrl->v_full[s]);
         tma_load_4d(vb + kHalf, mv, 64, 0, mg, w, &ctrl->v_full[s]);
       }
@@ -988,7 +1026,8 @@ int attn_tc_ctas() { return std::min(device_sm_count(), kTcMaxCtas); }
 cudaError_t launch_attn_tc(const AttnTcParams& prm, const void* q, const void* k_cache,
                            const void* v_cache, const void* draft_k, const void* draft_v,
                            cudaStream_t st) {
-  CUtensorMap tq, tk, tv, tdk, tdv;
+  CUtensorMap tq, tdk, tdv;
+  PageMaps pm;
   const uint64_t W1 = (uint64_t)prm.W1;
   {
     const cuuint64_t dims[4] = {kD, (cuuint64_t)prm.hq, W1, (cuuint64_t)prm.B};
@@ -1002,9 +1041,11 @@ cudaError_t launch_attn_tc(const AttnTcParams& prm, const void* q, const void* k
                                 (cuuint64_t)prm.num_pages};
     const cuuint64_t strides[3] = {kD * 2ull, kPage * kD * 2ull,
                                    (cuuint64_t)prm.hkv * kPage * kD * 2ull};
-    const cuuint32_t box[4] = {64, (cuuint32_t)kPage, 1, 1};
-    if (!encode_4d(&tk, k_cache, dims, strides, box)) return cudaErrorInvalidValue;
-    if (!encode_4d(&tv, v_cache, dims, strides, box)) return cudaErrorInvalidValue;
+    for (int i = 0; i < 4; ++i) {
+      const cuuint32_t box[4] = {64, (cuuint32_t)kPage, 1, 1u << i};
+      if (!encode_4d(&pm.k[i], k_cache, dims, strides, box)) return cudaErrorInvalidValue;
+      if (!encode_4d(&pm.v[i], v_cache, dims, strides, box)) return cudaErrorInvalidValue;
+    }
   }
   if (prm.draft) {
     // draft scratch [B, hkv, kmax, D]: one box = the 16-row draft page (rows
@@ -1016,8 +1057,8 @@ cudaError_t launch_attn_tc(const AttnTcParams& prm, const void* q, const void* k
     if (!encode_4d(&tdk, draft_k, dims, strides, box)) return cudaErrorInvalidValue;
     if (!encode_4d(&tdv, draft_v, dims, strides, box)) return cudaErrorInvalidValue;
   } else {
-    tdk = tk;
-    tdv = tv;
+    tdk = pm.k[0];
+    tdv = pm.v[0];
   }
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -1029,12 +1070,11 @@ cudaError_t launch_attn_tc(const AttnTcParams& prm, const void* q, const void* k
     if (e != cudaSuccess) return e;
     g_tc_attr_set.fetch_or(bit, std::memory_order_acq_rel);
   }
-  attn_tc_kernel<<<prm.nctas, kThreadsTC, kSmemTC, st>>>(tq, tk, tv, tdk, tdv, prm);
-  e = cudaGetLastError();
+  e = launch_pdl(attn_tc_kernel, dim3(prm.nctas), dim3(kThreadsTC), kSmemTC, st, tq, pm, tdk, tdv,
+                 prm);
   if (e != cudaSuccess) return e;
   const dim3 mgrid(prm.B * prm.hkv, (prm.G * prm.W1 + kMergeRows - 1) / kMergeRows);
-  attn_merge_kernel<<<mgrid, kMergeThreads, 0, st>>>(prm);
-  return cudaGetLastError();
+  return launch_pdl(attn_merge_kernel, mgrid, dim3(kMergeThreads), 0, st, prm);
 }
 
 size_t attn_tc_part_bound(int32_t group, int32_t w1) {

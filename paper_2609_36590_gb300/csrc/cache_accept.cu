@@ -18,6 +18,8 @@ __global__ void draft_append_kernel(int32_t hkv, int32_t D, int32_t kmax,
                                     const int32_t* __restrict__ draft_lens,
                                     uint16_t* __restrict__ draft_k,
                                     uint16_t* __restrict__ draft_v, int32_t* err) {
+  if (threadIdx.x == 0) pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x;
   const int chunks = D / 8;
   const int h = threadIdx.x / chunks, c = threadIdx.x - h * chunks;
@@ -42,6 +44,8 @@ __global__ void kv_append_kernel(int32_t hkv, int32_t D, int32_t kmax,
                                  const uint16_t* __restrict__ v_new,
                                  const int32_t* __restrict__ n_new,
                                  const int32_t* __restrict__ ctx_lens, int32_t* err) {
+  if (threadIdx.x == 0) pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x, j = blockIdx.y;
   const int chunks = D / 8;
   const int h = threadIdx.x / chunks, c = threadIdx.x - h * chunks;
@@ -79,6 +83,8 @@ __global__ void accept_kernel(int32_t B, int32_t kmax, const int32_t* __restrict
                               int32_t page_size, int32_t* __restrict__ ctx_lens,
                               int32_t* __restrict__ accepted, int32_t* __restrict__ tokens,
                               int32_t* __restrict__ slots, int32_t* err) {
+  if (threadIdx.x == 0) pdl_trigger();
+  pdl_wait();
   const int lane = threadIdx.x & 31;
   const int b = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (b >= B) return;
@@ -126,9 +132,8 @@ cudaError_t launch_draft_append(int32_t B, int32_t hkv, int32_t head_dim, int32_
                                 const int32_t* draft_lens, uint16_t* draft_k, uint16_t* draft_v,
                                 int32_t* err, cudaStream_t st) {
   const int threads = hkv * head_dim / 8;
-  draft_append_kernel<<<B, threads, 0, st>>>(hkv, head_dim, kmax, k_new, v_new, draft_lens,
-                                             draft_k, draft_v, err);
-  return cudaGetLastError();
+  return launch_pdl(draft_append_kernel, dim3(B), dim3(threads), 0, st, hkv, head_dim, kmax, k_new,
+                    v_new, draft_lens, draft_k, draft_v, err);
 }
 
 cudaError_t launch_kv_append(int32_t B, int32_t hkv, int32_t head_dim, int32_t kmax,
@@ -138,10 +143,8 @@ cudaError_t launch_kv_append(int32_t B, int32_t hkv, int32_t head_dim, int32_t k
                              const int32_t* ctx_lens, int32_t* err, cudaStream_t st) {
   const int threads = hkv * head_dim / 8;
   dim3 grid(B, kmax + 1);
-  kv_append_kernel<<<grid, threads, 0, st>>>(hkv, head_dim, kmax, k_cache, v_cache, page_table,
-                                             max_pages, num_pages, k_new, v_new, n_new,
-                                             ctx_lens, err);
-  return cudaGetLastError();
+  return launch_pdl(kv_append_kernel, grid, dim3(threads), 0, st, hkv, head_dim, kmax, k_cache,
+                    v_cache, page_table, max_pages, num_pages, k_new, v_new, n_new, ctx_lens, err);
 }
 
 cudaError_t launch_accept(int32_t B, int32_t kmax, const int32_t* draft_ids,
@@ -151,10 +154,9 @@ cudaError_t launch_accept(int32_t B, int32_t kmax, const int32_t* draft_ids,
                           int32_t* slots, int32_t* err, cudaStream_t st) {
   constexpr int kWarpsPerBlock = 4;
   const int grid = (B + kWarpsPerBlock - 1) / kWarpsPerBlock;
-  accept_kernel<<<grid, 32 * kWarpsPerBlock, 0, st>>>(B, kmax, draft_ids, target_ids, k_b,
-                                                      page_table, max_pages, page_size,
-                                                      ctx_lens, accepted, tokens, slots, err);
-  return cudaGetLastError();
+  return launch_pdl(accept_kernel, dim3(grid), dim3(32 * kWarpsPerBlock), 0, st, B, kmax,
+                    draft_ids, target_ids, k_b, page_table, max_pages, page_size, ctx_lens,
+                    accepted, tokens, slots, err);
 }
 
 }  // namespace seedk

@@ -9,6 +9,17 @@
 
 namespace seedk {
 
+// Programmatic dependent launch.  A kernel launched with launch_pdl may start
+// while the previous kernel of its stream is still finishing: it calls
+// pdl_trigger() early (letting the next kernel start in turn) and pdl_wait()
+// before its first access to global memory, which returns once the previous
+// kernel has completed and its writes are visible.  Both are no-ops for a
+// kernel launched normally.
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 constexpr int kPage = 16;                 // tokens per KV page (page_size)
 constexpr uint32_t kSpinLimit = 1u << 22; // polls before a wait gives up
 constexpr uint32_t kSuspendNs = 500000;   // per-try sleep bound of a suspending wait

@@ -5,10 +5,30 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <utility>
 
 namespace seedk {
 
 constexpr int kPageTokens = 16;   // tokens per KV page; the only page size built
+
+// Launch with programmatic stream serialisation: the kernel may begin while
+// the previous kernel of the stream finishes (it must call pdl_wait() before
+// touching global memory).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t st, Args&&... args) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 // Split-KV flash-decoding work description (see decode_attn.cu).
 struct DecodeParams {
