@@ -98,7 +98,7 @@ struct TileMeta {
 struct Ctrl {
   uint64_t k_full[kStagesTC], k_empty[kStagesTC];   // K ring
   uint64_t v_full[kStagesTC], v_empty[kStagesTC];   // V ring
-  uint64_t q_full, q_empty;
+  uint64_t q_full[2], q_empty[2];             // Q buffers (two when the rows fit 64)
   uint64_t meta_full[kMetaRing], meta_empty[kMetaRing];   // K warp -> V warp
   uint64_t s_full[2], p_full[2], o_full[2];   // per tile parity
   uint64_t stats_bar[4], orel_bar[4];         // per TMEM lane quarter
@@ -547,8 +547,10 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
       mbar_init(&ctrl->v_full[s], 1);
       mbar_init(&ctrl->v_empty[s], 1);
     }
-    mbar_init(&ctrl->q_full, 1);
-    mbar_init(&ctrl->q_empty, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&ctrl->q_full[i], 1);
+      mbar_init(&ctrl->q_empty[i], 1);
+    }
     for (int i = 0; i < kMetaRing; ++i) {
       mbar_init(&ctrl->meta_full[i], 1);
       mbar_init(&ctrl->meta_empty[i], 1);
@@ -575,6 +577,13 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
   tc_fence_after();
   const uint32_t tmem = ctrl->tmem_base;
   const int Rmax = p.G * p.W1;
+  // Q buffers.  With at most 64 query rows, two compact buffers (rows padded
+  // to 8, each head-dim half Rpad x 128 B) share the Q region, so that the Q
+  // of the next piece loads while S of the current one runs.  The MMA reads
+  // 128 rows from a buffer; rows past its Rpad are unused garbage rows.
+  const int Rpad = (Rmax + 7) & ~7;
+  const int nqb = Rpad <= 64 ? 2 : 1;
+  const uint32_t qhalf = nqb == 2 ? (uint32_t)Rpad * 128u : kHalf;
   // everything above touched only this CTA's shared and tensor memory
   pdl_wait();
 
@@ -638,7 +647,8 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
           ok = warp_wait(&ctrl->k_empty[s], ((tk / kStagesTC) - 1) & 1, ctrl, p.err);
         if (ok && tk >= kMetaRing)
           ok = warp_wait(&ctrl->meta_empty[mi], ((tk / kMetaRing) - 1) & 1, ctrl, p.err);
-        if (ok && t == t0 && uo > 0) ok = warp_wait(&ctrl->q_empty, (uo - 1) & 1, ctrl, p.err);
+        if (ok && t == t0 && uo >= nqb)
+          ok = warp_wait(&ctrl->q_empty[uo % nqb], ((uo / nqb) - 1) & 1, ctrl, p.err);
         if (!ok) break;
         if (lane < kPagesPerTile && t * kPagesPerTile + lane < sq.ncp &&
             (pid < 0 || pid >= p.num_pages)) {
@@ -669,9 +679,11 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
           m.dslot = dslot;
           mbar_arrive(&ctrl->meta_full[mi]);
           if (t == t0) {
-            mbar_arrive_expect_tx(&ctrl->q_full, 2u * 128u * (uint32_t)Rmax);
-            tma_load_4d(smem, &tm_q, 0, g * p.G, 0, b, &ctrl->q_full);
-            tma_load_4d(smem + kHalf, &tm_q, 64, g * p.G, 0, b, &ctrl->q_full);
+            const int qb = uo % nqb;
+            uint8_t* qd = smem + (size_t)qb * 2 * qhalf;
+            mbar_arrive_expect_tx(&ctrl->q_full[qb], 2u * 128u * (uint32_t)Rmax);
+            tma_load_4d(qd, &tm_q, 0, g * p.G, 0, b, &ctrl->q_full[qb]);
+            tma_load_4d(qd + qhalf, &tm_q, 64, g * p.G, 0, b, &ctrl->q_full[qb]);
           }
           mbar_arrive_expect_tx(&ctrl->k_full[s], (uint32_t)__popc(loads) * 2u * 2048u);
         }
@@ -750,7 +762,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
     // S(t) and S(t) after PV(t-2) (S(t) overwrites P(t-2) in the same TMEM
     // columns; one thread's MMAs execute in issue order).
     if (lane == 0) {
-      int ts = 0, tp = 0, uo = 0, t_end = 1 << 30;
+      int ts = 0, tp = 0, uo = 0, qcur = 0, t_end = 1 << 30;
       int k_of[kStagesTC];               // tile index within its unit, per stage
       uint32_t idle = 0;
       while (tp < t_end && !ctrl->abort_flag) {
@@ -765,9 +777,12 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
               did = true;
             } else {
               const int k = mt.k;
-              const bool q_ok = (k != 0) || mbar_test(&ctrl->q_full, uo & 1);
+              const bool q_ok = (k != 0) || mbar_test(&ctrl->q_full[uo % nqb], (uo / nqb) & 1);
               if (q_ok) {
-                if (k == 0) ++uo;
+                if (k == 0) {
+                  qcur = uo % nqb;
+                  ++uo;
+                }
                 k_of[s] = k;
                 tc_fence_after();
                 const uint32_t d = tmem + (uint32_t)(ts & 1) * kN;
@@ -775,13 +790,14 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
 #pragma unroll 1
                 for (int kk = 0; kk < kD / 16; ++kk) {
                   const uint32_t h = kk >> 2, off = (kk & 3) * 32;
-                  const uint64_t a = smem_desc_sw128(sbase + h * kHalf + off, 16, 1024);
+                  const uint64_t a =
+                      smem_desc_sw128(sbase + (uint32_t)(qcur * 2 + h) * qhalf + off, 16, 1024);
                   const uint64_t b = smem_desc_sw128(kb + h * kHalf + off, 16, 1024);
                   mma_ss(d, a, b, kIdescS, kk > 0);
                 }
                 mma_commit(&ctrl->s_full[ts & 1]);
                 mma_commit(&ctrl->k_empty[s]);
-                if (mt.k == mt.ntu - 1) mma_commit(&ctrl->q_empty);
+                if (mt.k == mt.ntu - 1) mma_commit(&ctrl->q_empty[qcur]);
                 ++ts;
                 did = true;
               }
