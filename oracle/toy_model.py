@@ -180,3 +180,105 @@ def seed_greedy(model: ToyLM, prompt, n_new: int, d: int, drafter: str = "model"
         L = int(new_L[0])
         rounds.append(n)
     return out[:n_new], rounds
+
+
+def seed_tree_greedy(model: ToyLM, prompt, n_new: int, depth: int, width: int,
+                     drafter: str = "model", reference=None, page_size: int = 4,
+                     page_seed: int = 0, mistake: str | None = None):
+    """SEED with a draft tree and tree-based verification (Sec. D.1).
+
+    Each round drafts a main branch of `depth` tokens with f_dec (as in Alg. 2);
+    at every step the node being extended gets `width` children, the drafter's
+    top-`width` distinct tokens, and the top-1 child continues the branch.
+    drafter 'perfect' / 'adversarial' force the top-1 child to the reference
+    token / a wrong token (its siblings stay the drafter's next choices).  All
+    nodes are verified in one pass with the tree mask; the tree is walked
+    greedily; the accepted path's rows are compacted into place.
+
+    mistake (planted, for the tests): 'causal' lets every node see all earlier
+    packed rows (siblings included); 'nocompact' skips moving the accepted
+    rows.  Returns (tokens, accepted count per round).
+    """
+    from . import tree as _tree
+
+    L = len(prompt) - 1
+    pending = int(prompt[-1])
+    n_nodes = 1 + depth * width
+    cap = len(prompt) + n_new + n_nodes + 2
+    n_pages = -(-cap // page_size)
+    pt = np.random.default_rng(page_seed).permutation(n_pages).astype(np.int32)
+    shape = (n_pages, model.hkv, page_size, model.hd)
+    kc = [np.full(shape, np.nan) for _ in range(model.n_layers)]
+    vc = [np.full(shape, np.nan) for _ in range(model.n_layers)]
+    if L > 0:
+        _, ks, vs = model.forward_dense(list(prompt[:L]))
+        for l in range(model.n_layers):
+            _cache.write_rows(kc[l], pt, 0, ks[l])
+            _cache.write_rows(vc[l], pt, 0, vs[l])
+
+    dec = range(model.split, model.n_layers)
+    out, rounds = [], []
+    while len(out) < n_new:
+        # ---- drafting: the main branch, with `width` children per step
+        tok, parent = [pending], [-1]
+        main = 0
+        dk = {l: [] for l in dec}
+        dv = {l: [] for l in dec}
+        for i in range(1, depth + 1):
+            h = model.embed([tok[main]], [L + i - 1])
+            for l in dec:
+                q, k, v = model.qkv(l, h)
+                dk[l].append(k[0])
+                dv[l].append(v[0])
+                o, _ = _attn.draft_attention_seq(
+                    q[0], _cache.gather_rows(kc[l], pt, L), _cache.gather_rows(vc[l], pt, L),
+                    np.stack(dk[l]), np.stack(dv[l]), model.scale)
+                h = model.post(l, h, o[None])
+            order = [int(t) for t in np.argsort(-model.logits(h)[0], kind="stable")]
+            ref_i = len(out) + i - 1
+            first = None
+            if drafter == "perfect" and reference is not None and ref_i < len(reference):
+                first = int(reference[ref_i])
+            elif drafter == "adversarial" and reference is not None and ref_i < len(reference):
+                first = (int(reference[ref_i]) + 1) % model.vocab
+            kids = ([first] if first is not None else []) + [t for t in order if t != first]
+            kids = kids[:width]
+            base = len(tok)
+            for t in kids:
+                tok.append(t)
+                parent.append(main)
+            main = base
+        n = len(tok)
+
+        # ---- verification: all nodes in one pass with the tree mask
+        dep = _tree.depths(parent)
+        H = model.embed(tok, L + dep)
+        pmask = list(range(-1, n - 1)) if mistake == "causal" else parent
+        for l in range(model.n_layers):
+            q, k, v = model.qkv(l, H)
+            _cache.write_rows(kc[l], pt, L, k)
+            _cache.write_rows(vc[l], pt, L, v)
+            o, _ = _tree.tree_verify_attention_seq(
+                q, _cache.gather_rows(kc[l], pt, L + n), _cache.gather_rows(vc[l], pt, L + n),
+                L, pmask, model.scale)
+            H = model.post(l, H, o)
+        target = np.argmax(model.logits(H), axis=1)
+
+        # ---- greedy walk, commit of the accepted path
+        acc, tokens, path, _, new_L = _tree.tree_accept_commit(
+            np.array([tok]), np.array([parent]), [n], target[None, :], [L], pt[None, :],
+            page_size)
+        m = int(acc[0])
+        for l in range(model.n_layers):
+            if mistake != "nocompact":
+                for c in (kc[l], vc[l]):
+                    rows = _cache.gather_rows(c, pt, L + n)
+                    rows = _tree.compact_path(rows, L, path[0], m)
+                    _cache.write_rows(c, pt, L, rows[L:L + m + 1])
+            _cache.poison_from(kc[l], pt, int(new_L[0]), n_pages * page_size)
+            _cache.poison_from(vc[l], pt, int(new_L[0]), n_pages * page_size)
+        out.extend(int(t) for t in tokens[0, :m + 1])
+        pending = int(tokens[0, m])
+        L = int(new_L[0])
+        rounds.append(m)
+    return out[:n_new], rounds
