@@ -12,8 +12,13 @@ the paper (SEED: Self-Speculative Decoding via Implicit Encoder-Decoder):
   Sec. 3).
 * ``accept``     -- greedy longest-prefix acceptance, bonus token and the
   commit/rollback of cache rows (Alg. 2, acceptance and truncation steps).
-* ``toy_model``  -- a tiny float64 transformer running Alg. 2 end to end and
-  plain greedy decoding, for the exactness property of Sec. 4.1.
+* ``tree``       -- tree-based verification (Sec. D.1): the tree mask (each
+  candidate sees the verified prefix and its own ancestral path), the greedy
+  walk from the root with its bonus token, and the compaction of the accepted
+  path's cache rows.
+* ``toy_model``  -- a tiny float64 transformer running Alg. 2 end to end (with
+  a linear draft or a draft tree) and plain greedy decoding, for the
+  exactness property of Sec. 4.1.
 
 Only ``tests/``, ``__graft_entry__.smoke()`` and the ``cpu_baseline`` /
 ``--impl reference`` legs of ``bench.py`` may import this package.  It shares
