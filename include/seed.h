@@ -45,8 +45,8 @@
 extern "C" {
 #endif
 
-#define SEED_ABI_VERSION 1
-#define SEED_MAX_KMAX 16        /* largest supported draft length d */
+#define SEED_ABI_VERSION 2
+#define SEED_MAX_KMAX 31        /* largest supported draft length d (32 rows per sequence) */
 
 typedef enum {
   SEED_OK = 0,
@@ -67,6 +67,7 @@ typedef enum {
 #define SEED_DEVERR_KB        16  /* k_b outside [0, kmax]                          */
 #define SEED_DEVERR_WORKSPACE 32  /* more work units than the workspace holds       */
 #define SEED_DEVERR_TIMEOUT   64  /* a bounded on-chip wait gave up (never expected) */
+#define SEED_DEVERR_TREE      128 /* a draft tree's parents or accepted path are invalid */
 
 /* Shapes of one model's attention.  Supported: head_dim in {64, 128};
  * hq / hkv in {1, 2, 4, 8}; page_size == 16; 1 <= kmax <= SEED_MAX_KMAX.
@@ -190,6 +191,77 @@ seed_status_t seed_accept_commit(int32_t batch, int32_t kmax, const int32_t* dra
                                  int32_t page_size, int32_t* ctx_lens, int32_t* accepted,
                                  int32_t* tokens, int32_t* committed_slots,
                                  int32_t* err_flag, void* stream);
+
+/* ------------------------------------------------------------------------
+ * Tree-based verification (Sec. D.1).  The drafter proposes a tree of
+ * candidates instead of one chain; the verifier checks all of them in one
+ * pass, each candidate seeing the verified prefix and its own ancestral path
+ * only; the tree is then walked greedily from the root and the cache keeps
+ * the accepted path.
+ *
+ * A tree of sequence b has n_nodes[b] <= kmax + 1 nodes, numbered so that
+ * every node comes after its parent.  Node 0 is the root: the last verified
+ * token (X_draft[0] of the linear case), whose row is not in the cache yet.
+ * Node i's K/V row is written with seed_kv_append (n_new = n_nodes) at packed
+ * position ctx_lens[b] + i; its model position, for position embeddings, is
+ * ctx_lens[b] + depth(i).  One round is:
+ *   per layer:  seed_kv_append, seed_tree_verify_attn
+ *   then:       seed_tree_accept_commit (once), seed_tree_kv_compact (per layer)
+ * ------------------------------------------------------------------------ */
+
+/* Verify attention over a draft tree (Sec. D.1, tree-structured mask): node
+ * j (j < n_nodes[b]) of sequence b attends to cache rows 0 .. ctx_lens[b]-1
+ * and to the packed rows ctx_lens[b] + a of the nodes a whose bit is set in
+ * anc[b, j] (its ancestors; the node's own bit is always added, bits at or
+ * past n_nodes[b] are ignored).
+ *   q         bf16 [batch, kmax+1, hq, head_dim] (row j = node j)
+ *   n_nodes   int32 [batch] in [0, kmax+1] (0 skips the sequence)
+ *   anc       uint32 [batch, kmax+1]: bit a of anc[b, j] = node a is an
+ *             ancestor of node j
+ *   others    as seed_verify_attn (same workspace size)
+ * Built for head_dim 128 with (hq/hkv) * (kmax+1) <= 128; other shapes
+ * return SEED_ERR_UNSUPPORTED.
+ * Device errors: SEED_DEVERR_CTX_LEN, _NQ, _PAGE. */
+seed_status_t seed_tree_verify_attn(const seed_cfg_t* cfg, int32_t batch, const void* q,
+                                    const int32_t* n_nodes, const uint32_t* anc,
+                                    seed_kv_t kv, const int32_t* ctx_lens,
+                                    float* out, float* lse, void* ws, size_t ws_bytes,
+                                    int32_t* err_flag, void* stream);
+
+/* Greedy acceptance over a draft tree (Sec. D.1): from the root, take the
+ * child of the current node whose token equals target_ids at the current
+ * node (the lowest node index if several do), until no child matches.  n_b =
+ * accepted drafts; tokens[b] = their tokens then the bonus target_ids[b, last
+ * accepted node]; path[b, d] = node at depth d of the accepted path
+ * (path[b, 0] = 0); committed_slots = slots of positions ctx_lens[b] ..
+ * ctx_lens[b] + n_b (where seed_tree_kv_compact puts the path's rows);
+ * ctx_lens[b] += n_b + 1.
+ *   tok         int32 [batch, kmax+1]: node tokens (tok[b, 0] = root)
+ *   parent      int32 [batch, kmax+1]: parent[b, i] < i for 1 <= i < n_nodes
+ *   n_nodes     int32 [batch] in [1, kmax+1]
+ *   target_ids  int32 [batch, kmax+1]: the verifier's argmax at each node
+ *   accepted    int32 [batch]; tokens, path, committed_slots int32
+ *               [batch, kmax+1], -1 past the used entries
+ * Device errors: SEED_DEVERR_NQ (n_nodes), _TREE (a parent not before its
+ * node), _CTX_LEN (the tree's rows past capacity); that sequence is then left
+ * unchanged. */
+seed_status_t seed_tree_accept_commit(int32_t batch, int32_t kmax, const int32_t* tok,
+                                      const int32_t* parent, const int32_t* n_nodes,
+                                      const int32_t* target_ids, const int32_t* page_table,
+                                      int32_t max_pages, int32_t page_size, int32_t* ctx_lens,
+                                      int32_t* accepted, int32_t* tokens, int32_t* path,
+                                      int32_t* committed_slots, int32_t* err_flag,
+                                      void* stream);
+
+/* Cache side of the tree commit, per layer: moves the rows of the accepted
+ * path from their packed positions L + path[b, d] to L + d (d = 1..n_b), with
+ * L = ctx_lens[b] - accepted[b] - 1 (ctx_lens and accepted as
+ * seed_tree_accept_commit left them).
+ * Device errors: SEED_DEVERR_TREE (path not increasing from depth d on, or
+ * past capacity), _CTX_LEN, _PAGE. */
+seed_status_t seed_tree_kv_compact(const seed_cfg_t* cfg, int32_t batch, seed_kv_t kv,
+                                   const int32_t* path, const int32_t* accepted,
+                                   const int32_t* ctx_lens, int32_t* err_flag, void* stream);
 
 /* ------------------------------------------------------------------------
  * Library convenience with no counterpart in the paper: verify attention

@@ -9,7 +9,8 @@ every entry point fails loudly when the library has not been built.
 Entry points carry the C names: seed_workspace_bytes, seed_draft_kv_append,
 seed_draft_attn, seed_kv_append, seed_verify_attn, seed_accept_commit, and
 seed_verify_attn_noalloc (verify attention on the library's built-in scratch,
-for callers that cannot provide a workspace).
+for callers that cannot provide a workspace), and the tree-verification calls
+seed_tree_verify_attn, seed_tree_accept_commit, seed_tree_kv_compact.
 """
 
 from __future__ import annotations
@@ -27,8 +28,8 @@ SEED_OK = 0
 SEED_ERR_SCRATCH_LIMIT = 7
 NOALLOC_SCRATCH_BYTES = 32 << 20   # SEED_NOALLOC_SCRATCH_BYTES of seed.h
 DEVERR = {1: "ctx_len", 2: "draft_len", 4: "n_q", 8: "page", 16: "k_b", 32: "workspace",
-          64: "timeout"}
-MAX_KMAX = 16
+          64: "timeout", 128: "tree"}
+MAX_KMAX = 31
 
 
 class _Cfg(ctypes.Structure):
@@ -56,6 +57,11 @@ _SIGS = {
     "seed_accept_commit": (_I, [_I, _I, _P, _P, _P, _P, _I, _I, _P, _P, _P, _P, _P, _P]),
     "seed_verify_attn_noalloc": (_I, [ctypes.POINTER(_Cfg), _I, _P, _P, _KV, _P, _P, _P, _P,
                                       _P]),
+    "seed_tree_verify_attn": (_I, [ctypes.POINTER(_Cfg), _I, _P, _P, _P, _KV, _P, _P, _P, _P,
+                                   ctypes.c_size_t, _P, _P]),
+    "seed_tree_accept_commit": (_I, [_I, _I, _P, _P, _P, _P, _P, _I, _I, _P, _P, _P, _P, _P,
+                                     _P, _P]),
+    "seed_tree_kv_compact": (_I, [ctypes.POINTER(_Cfg), _I, _KV, _P, _P, _P, _P, _P]),
 }
 
 
@@ -242,6 +248,59 @@ def seed_verify_attn_noalloc(cfg: SeedConfig, q, n_q, kv: PagedKV, ctx_lens, out
         _t(ctx_lens, torch.int32, (B,), "ctx_lens"),
         _t(out, torch.float32, (B, W, cfg.hq, cfg.head_dim), "out"),
         _t(lse, torch.float32, (B, W, cfg.hq), "lse") if lse is not None else None,
+        _t(err, torch.int32, (1,), "err"), _stream(stream)))
+
+
+def seed_tree_verify_attn(cfg: SeedConfig, q, n_nodes, anc, kv: PagedKV, ctx_lens, out, lse, ws,
+                          err, stream=None) -> None:
+    """Verify attention over draft trees (tree-structured mask); anc is int32
+    holding the uint32 ancestor bit masks [B, kmax+1]."""
+    B = q.shape[0]
+    c = cfg.c()
+    W = cfg.kmax + 1
+    _check(_lib.seed_tree_verify_attn(
+        ctypes.byref(c), B,
+        _t(q, torch.bfloat16, (B, W, cfg.hq, cfg.head_dim), "q"),
+        _t(n_nodes, torch.int32, (B,), "n_nodes"),
+        _t(anc, torch.int32, (B, W), "anc"),
+        _kv_checked(cfg, kv, B),
+        _t(ctx_lens, torch.int32, (B,), "ctx_lens"),
+        _t(out, torch.float32, (B, W, cfg.hq, cfg.head_dim), "out"),
+        _t(lse, torch.float32, (B, W, cfg.hq), "lse") if lse is not None else None,
+        _t(ws, torch.uint8, None, "ws"), ws.numel(),
+        _t(err, torch.int32, (1,), "err"), _stream(stream)))
+
+
+def seed_tree_accept_commit(kmax: int, tok, parent, n_nodes, target_ids, page_table,
+                            page_size: int, ctx_lens, accepted, tokens, path, committed_slots,
+                            err, stream=None) -> None:
+    B = n_nodes.shape[0]
+    W = kmax + 1
+    _check(_lib.seed_tree_accept_commit(
+        B, kmax,
+        _t(tok, torch.int32, (B, W), "tok"),
+        _t(parent, torch.int32, (B, W), "parent"),
+        _t(n_nodes, torch.int32, (B,), "n_nodes"),
+        _t(target_ids, torch.int32, (B, W), "target_ids"),
+        _t(page_table, torch.int32, (B, page_table.shape[1]), "page_table"),
+        page_table.shape[1], page_size,
+        _t(ctx_lens, torch.int32, (B,), "ctx_lens"),
+        _t(accepted, torch.int32, (B,), "accepted"),
+        _t(tokens, torch.int32, (B, W), "tokens"),
+        _t(path, torch.int32, (B, W), "path"),
+        _t(committed_slots, torch.int32, (B, W), "committed_slots"),
+        _t(err, torch.int32, (1,), "err"), _stream(stream)))
+
+
+def seed_tree_kv_compact(cfg: SeedConfig, kv: PagedKV, path, accepted, ctx_lens, err,
+                         stream=None) -> None:
+    B = accepted.shape[0]
+    c = cfg.c()
+    _check(_lib.seed_tree_kv_compact(
+        ctypes.byref(c), B, _kv_checked(cfg, kv, B),
+        _t(path, torch.int32, (B, cfg.kmax + 1), "path"),
+        _t(accepted, torch.int32, (B,), "accepted"),
+        _t(ctx_lens, torch.int32, (B,), "ctx_lens"),
         _t(err, torch.int32, (1,), "err"), _stream(stream)))
 
 

@@ -273,8 +273,11 @@ __device__ __noinline__ void next_seq(const AttnTcParams& p, int lane, SeqWin& w
 // ------------------------------------------------------------- the kernel
 // One softmax row: the visible columns of a tile for query j are the cache
 // columns c <= lim (c < dcol) and the draft columns dcol <= c < dend.
+// For a tree verify (Sec. D.1) the cache columns of the tree's packed rows
+// start at column tb, and bit a of tm makes packed row a visible.
 struct ColMask {
-  int dcol, dend, lim;
+  int dcol, dend, lim, tb;
+  uint32_t tm;
   // bit i set <=> column c0 + i is visible
   __device__ __forceinline__ uint32_t bits(int c0) const {
     const int nc = min(max(min(lim, dcol - 1) - c0 + 1, 0), 32);
@@ -282,7 +285,9 @@ struct ColMask {
     const uint32_t mc = nc == 32 ? 0xffffffffu : ((1u << nc) - 1u);
     const uint32_t mh = hi == 32 ? 0xffffffffu : ((1u << hi) - 1u);
     const uint32_t ml = lo == 32 ? 0xffffffffu : ((1u << lo) - 1u);
-    return mc | (mh & ~ml);
+    const int off = c0 - tb;   // packed row seen at column c0
+    const uint32_t mt = (off >= 32 || off <= -32) ? 0u : off >= 0 ? (tm >> off) : (tm << -off);
+    return mc | (mh & ~ml) | mt;
   }
 };
 
@@ -863,6 +868,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
     const int nqa = min(4, (p.G * p.W1 + 31) / 32);   // lane quarters in use
     const float c2 = p.scale_log2;
     float m_used = -INFINITY, l = 0.f;
+    uint32_t tmask = 0u;
     int xcnt = 0;
     bool pend_rel = false;
     // (every wait below gives up once another role has aborted; the lanes
@@ -876,17 +882,31 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
       const TileMeta m = ctrl->meta[t % kMetaRing];
       tc_fence_after();
       const bool first_own = m.k < 2;
+      const int R = m.nq * p.G;
+      const int j = row / p.G;
       if (first_own) {
         m_used = -INFINITY;
         l = 0.f;
+        // tree verify: this row's ancestors among the packed rows, clamped to
+        // the tree's nodes, the node itself always included
+        if (p.anc != nullptr && row < R) {
+          const uint32_t below = m.nq >= 32 ? 0xffffffffu : ((1u << m.nq) - 1u);
+          tmask = (__ldg(p.anc + (size_t)m.b * p.W1 + j) | (1u << j)) & below;
+        }
       }
-      const int R = m.nq * p.G;
-      const int j = row / p.G;
       const bool warp_active = q4 * 32 < R;
       ColMask cm;
       cm.dcol = (m.ncp - m.tile * kPagesPerTile) * kPage;   // first draft column
       cm.dend = cm.dcol + m.nd;
-      cm.lim = m.lim0 + j - m.tile * kN;                     // cache columns <= lim visible
+      if (p.anc == nullptr) {
+        cm.lim = m.lim0 + j - m.tile * kN;                   // cache columns <= lim visible
+        cm.tb = 0;
+        cm.tm = 0u;
+      } else {
+        cm.lim = m.lim0 - 1 - m.tile * kN;                   // the committed rows
+        cm.tb = m.lim0 - m.tile * kN;                        // packed row 0
+        cm.tm = tmask;
+      }
       bool resc = false;
       float fo = 1.f;
       const uint32_t scol = tmem + lane_off + (uint32_t)par * kN;

@@ -127,6 +127,123 @@ __global__ void accept_kernel(int32_t B, int32_t kmax, const int32_t* __restrict
 
 }  // namespace
 
+// Tree acceptance (Sec. D.1): one warp per sequence, lane i = node i of the
+// linearised tree (at most 32 nodes).  From the root, the walk takes the
+// lowest-index child whose token equals the verifier's argmax at the current
+// node, until no child matches; the bonus token is the argmax at the last
+// accepted node.  Outputs follow seed_accept_commit, plus the accepted path.
+__global__ void tree_accept_kernel(int32_t B, int32_t kmax, const int32_t* __restrict__ tok,
+                                   const int32_t* __restrict__ parent,
+                                   const int32_t* __restrict__ n_nodes,
+                                   const int32_t* __restrict__ target_ids,
+                                   const int32_t* __restrict__ page_table, int32_t max_pages,
+                                   int32_t page_size, int32_t* __restrict__ ctx_lens,
+                                   int32_t* __restrict__ accepted, int32_t* __restrict__ tokens,
+                                   int32_t* __restrict__ path, int32_t* __restrict__ slots,
+                                   int32_t* err) {
+  if (threadIdx.x == 0) pdl_trigger();
+  pdl_wait();
+  const int lane = threadIdx.x & 31;
+  const int b = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (b >= B) return;
+  const int W = kmax + 1;
+  const size_t row = (size_t)b * W;
+  const int n = n_nodes[b];
+  const int L = ctx_lens[b];
+  const bool bad_n = n < 1 || n > W;
+  const bool in = !bad_n && lane < n;
+  const int par = (in && lane > 0) ? parent[row + lane] : -1;
+  const int t = in ? tok[row + lane] : -1;
+  const int tg = in ? target_ids[row + lane] : -1;
+  const bool bad_par = __any_sync(0xffffffffu, in && lane > 0 && (par < 0 || par >= lane));
+  const long long cap = (long long)max_pages * page_size;
+  const bool bad_len = L < 0 || (!bad_n && (long long)L + n > cap);
+  if (bad_n || bad_par || bad_len) {
+    if (lane == 0)
+      raise_err(err, bad_n ? SEED_DEVERR_NQ : bad_par ? SEED_DEVERR_TREE : SEED_DEVERR_CTX_LEN);
+    return;
+  }
+  // the walk; lane d keeps the node at depth d of the accepted path
+  int cur = 0, depth = 0, mypath = lane == 0 ? 0 : -1;
+  for (int it = 0; it < 32; ++it) {
+    const int want = __shfl_sync(0xffffffffu, tg, cur);
+    const unsigned m = __ballot_sync(0xffffffffu, in && lane > 0 && par == cur && t == want);
+    if (m == 0u) break;
+    cur = __ffs((int)m) - 1;
+    ++depth;
+    if (lane == depth) mypath = cur;
+  }
+  const int bonus = __shfl_sync(0xffffffffu, tg, cur);
+  const int next = __shfl_sync(0xffffffffu, mypath, (lane + 1) & 31);   // path[lane + 1]
+  const int tnext = __shfl_sync(0xffffffffu, t, next < 0 ? 0 : next);
+  if (lane < W) {
+    int out_tok = -1, out_slot = -1;
+    if (lane < depth) out_tok = tnext;
+    else if (lane == depth) out_tok = bonus;
+    if (lane <= depth) {
+      const int pos = L + lane;
+      out_slot = page_table[(size_t)b * max_pages + pos / page_size] * page_size + pos % page_size;
+    }
+    tokens[row + lane] = out_tok;
+    slots[row + lane] = out_slot;
+    path[row + lane] = lane <= depth ? mypath : -1;
+  }
+  if (lane == 0) {
+    accepted[b] = depth;
+    ctx_lens[b] = L + depth + 1;
+  }
+}
+
+// Commit of a tree's accepted path in one layer's cache: the row of the node at
+// depth d moves from packed position L + path[d] to L + d (d = 1..n), one
+// depth at a time (a later move never reads a row an earlier one wrote).
+// grid (batch), block hkv * D / 8 threads; runs after tree_accept_kernel, whose
+// updated ctx_lens and accepted give L = ctx_lens - accepted - 1.
+__global__ void tree_compact_kernel(int32_t hkv, int32_t D, int32_t kmax,
+                                    uint16_t* __restrict__ k_cache,
+                                    uint16_t* __restrict__ v_cache,
+                                    const int32_t* __restrict__ page_table, int32_t max_pages,
+                                    int32_t num_pages, const int32_t* __restrict__ path,
+                                    const int32_t* __restrict__ accepted,
+                                    const int32_t* __restrict__ ctx_lens, int32_t* err) {
+  if (threadIdx.x == 0) pdl_trigger();
+  pdl_wait();
+  const int b = blockIdx.x;
+  const int chunks = D / 8;
+  const int h = threadIdx.x / chunks, c = threadIdx.x - h * chunks;
+  const int W = kmax + 1;
+  const int n = accepted[b];
+  const int L = ctx_lens[b] - n - 1;
+  if (n < 0 || n > kmax || L < 0) {
+    if (threadIdx.x == 0) raise_err(err, n < 0 || n > kmax ? SEED_DEVERR_TREE : SEED_DEVERR_CTX_LEN);
+    return;
+  }
+  const long long cap = (long long)max_pages * kPage;
+  for (int d = 1; d <= n; ++d) {
+    const int pd = path[(size_t)b * W + d];
+    if (pd < d || pd > kmax || (long long)L + pd >= cap) {
+      if (threadIdx.x == 0) raise_err(err, SEED_DEVERR_TREE);
+      return;
+    }
+  }
+  for (int d = 1; d <= n; ++d) {
+    const int src = L + path[(size_t)b * W + d], dst = L + d;
+    if (src != dst && h < hkv) {
+      const int ps = page_table[(size_t)b * max_pages + src / kPage];
+      const int pdst = page_table[(size_t)b * max_pages + dst / kPage];
+      if (ps < 0 || ps >= num_pages || pdst < 0 || pdst >= num_pages) {
+        raise_err(err, SEED_DEVERR_PAGE);
+      } else {
+        const size_t so = (((size_t)ps * hkv + h) * kPage + src % kPage) * D + c * 8;
+        const size_t dof = (((size_t)pdst * hkv + h) * kPage + dst % kPage) * D + c * 8;
+        *reinterpret_cast<uint4*>(k_cache + dof) = *reinterpret_cast<const uint4*>(k_cache + so);
+        *reinterpret_cast<uint4*>(v_cache + dof) = *reinterpret_cast<const uint4*>(v_cache + so);
+      }
+    }
+    __syncthreads();
+  }
+}
+
 cudaError_t launch_draft_append(int32_t B, int32_t hkv, int32_t head_dim, int32_t kmax,
                                 const uint16_t* k_new, const uint16_t* v_new,
                                 const int32_t* draft_lens, uint16_t* draft_k, uint16_t* draft_v,
@@ -157,6 +274,29 @@ cudaError_t launch_accept(int32_t B, int32_t kmax, const int32_t* draft_ids,
   return launch_pdl(accept_kernel, dim3(grid), dim3(32 * kWarpsPerBlock), 0, st, B, kmax,
                     draft_ids, target_ids, k_b, page_table, max_pages, page_size, ctx_lens,
                     accepted, tokens, slots, err);
+}
+
+cudaError_t launch_tree_accept(int32_t B, int32_t kmax, const int32_t* tok, const int32_t* parent,
+                               const int32_t* n_nodes, const int32_t* target_ids,
+                               const int32_t* page_table, int32_t max_pages, int32_t page_size,
+                               int32_t* ctx_lens, int32_t* accepted, int32_t* tokens,
+                               int32_t* path, int32_t* slots, int32_t* err, cudaStream_t st) {
+  constexpr int kWarpsPerBlock = 4;
+  const int grid = (B + kWarpsPerBlock - 1) / kWarpsPerBlock;
+  return launch_pdl(tree_accept_kernel, dim3(grid), dim3(32 * kWarpsPerBlock), 0, st, B, kmax,
+                    tok, parent, n_nodes, target_ids, page_table, max_pages, page_size, ctx_lens,
+                    accepted, tokens, path, slots, err);
+}
+
+cudaError_t launch_tree_compact(int32_t B, int32_t hkv, int32_t head_dim, int32_t kmax,
+                                uint16_t* k_cache, uint16_t* v_cache, const int32_t* page_table,
+                                int32_t max_pages, int32_t num_pages, const int32_t* path,
+                                const int32_t* accepted, const int32_t* ctx_lens, int32_t* err,
+                                cudaStream_t st) {
+  const int threads = hkv * head_dim / 8;
+  return launch_pdl(tree_compact_kernel, dim3(B), dim3(threads), 0, st, hkv, head_dim, kmax,
+                    k_cache, v_cache, page_table, max_pages, num_pages, path, accepted, ctx_lens,
+                    err);
 }
 
 }  // namespace seedk

@@ -87,6 +87,18 @@ cudaError_t launch_accept(int32_t B, int32_t kmax, const int32_t* draft_ids,
                           int32_t* ctx_lens, int32_t* accepted, int32_t* tokens,
                           int32_t* slots, int32_t* err, cudaStream_t st);
 
+cudaError_t launch_tree_accept(int32_t B, int32_t kmax, const int32_t* tok, const int32_t* parent,
+                               const int32_t* n_nodes, const int32_t* target_ids,
+                               const int32_t* page_table, int32_t max_pages, int32_t page_size,
+                               int32_t* ctx_lens, int32_t* accepted, int32_t* tokens,
+                               int32_t* path, int32_t* slots, int32_t* err, cudaStream_t st);
+
+cudaError_t launch_tree_compact(int32_t B, int32_t hkv, int32_t head_dim, int32_t kmax,
+                                uint16_t* k_cache, uint16_t* v_cache, const int32_t* page_table,
+                                int32_t max_pages, int32_t num_pages, const int32_t* path,
+                                const int32_t* accepted, const int32_t* ctx_lens, int32_t* err,
+                                cudaStream_t st);
+
 int device_sm_count();
 
 // Tensor-core draft and verify attention (attn_tc.cu).
@@ -98,6 +110,7 @@ struct AttnTcParams {
   int32_t num_pages;
   const int32_t* ctx_lens;    // [B]
   const int32_t* aux;         // verify: n_q [B]; draft: draft_lens [B]
+  const uint32_t* anc;        // tree verify: [B, W1] ancestor masks; else null
   float* out;                 // f32 [B, W1, hq, 128]
   float* lse;                 // f32 [B, W1, hq] or null
   float* part;                // partial records: two slots per CTA

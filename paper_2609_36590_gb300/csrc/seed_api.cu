@@ -95,7 +95,8 @@ seed_status_t run_decode(const seed_cfg_t* cfg, int32_t batch, bool verify, cons
 seed_status_t run_attn_tc(const seed_cfg_t* cfg, int32_t batch, bool draft, const void* q,
                           const int32_t* aux, const seed_kv_t& kv, const void* draft_k,
                           const void* draft_v, const int32_t* ctx_lens, float* out, float* lse,
-                          void* ws, size_t ws_bytes, int32_t* err, void* stream) {
+                          void* ws, size_t ws_bytes, int32_t* err, void* stream,
+                          const uint32_t* anc = nullptr) {
   const int G = cfg->hq / cfg->hkv;
   const int W1 = draft ? 1 : cfg->kmax + 1;
   const size_t cb = kSchedBytes + counters_bytes(cfg, batch);
@@ -108,6 +109,7 @@ seed_status_t run_attn_tc(const seed_cfg_t* cfg, int32_t batch, bool draft, cons
   p.num_pages = kv.num_pages;
   p.ctx_lens = ctx_lens;
   p.aux = aux;
+  p.anc = anc;
   p.out = out;
   p.lse = lse;
   p.part = reinterpret_cast<float*>(static_cast<char*>(ws) + cb);
@@ -236,6 +238,24 @@ seed_status_t seed_verify_attn(const seed_cfg_t* cfg, int32_t batch, const void*
                     ws_bytes, err_flag, stream);
 }
 
+seed_status_t seed_tree_verify_attn(const seed_cfg_t* cfg, int32_t batch, const void* q,
+                                    const int32_t* n_nodes, const uint32_t* anc, seed_kv_t kv,
+                                    const int32_t* ctx_lens, float* out, float* lse, void* ws,
+                                    size_t ws_bytes, int32_t* err_flag, void* stream) {
+  seed_status_t st = check_cfg(cfg);
+  if (st != SEED_OK) return st;
+  if (batch < 0) return SEED_ERR_SHAPE;
+  if (!seedk::attn_tc_supported(cfg->head_dim, cfg->hq / cfg->hkv, cfg->kmax + 1))
+    return SEED_ERR_UNSUPPORTED;
+  if (batch == 0) return SEED_OK;
+  if (!q || !n_nodes || !anc || !ctx_lens || !out || !ws || !err_flag) return SEED_ERR_NULL;
+  if ((st = check_kv(kv)) != SEED_OK) return st;
+  if (misaligned16(q) || misaligned16(kv.k) || misaligned16(kv.v)) return SEED_ERR_RANGE;
+  if ((reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)) != 0) return SEED_ERR_WORKSPACE;
+  return run_attn_tc(cfg, batch, false, q, n_nodes, kv, nullptr, nullptr, ctx_lens, out, lse, ws,
+                     ws_bytes, err_flag, stream, anc);
+}
+
 seed_status_t seed_accept_commit(int32_t batch, int32_t kmax, const int32_t* draft_ids,
                                  const int32_t* target_ids, const int32_t* k_b,
                                  const int32_t* page_table, int32_t max_pages,
@@ -253,6 +273,42 @@ seed_status_t seed_accept_commit(int32_t batch, int32_t kmax, const int32_t* dra
                                      max_pages, page_size, ctx_lens, accepted, tokens,
                                      committed_slots, err_flag,
                                      static_cast<cudaStream_t>(stream)));
+}
+
+seed_status_t seed_tree_accept_commit(int32_t batch, int32_t kmax, const int32_t* tok,
+                                      const int32_t* parent, const int32_t* n_nodes,
+                                      const int32_t* target_ids, const int32_t* page_table,
+                                      int32_t max_pages, int32_t page_size, int32_t* ctx_lens,
+                                      int32_t* accepted, int32_t* tokens, int32_t* path,
+                                      int32_t* committed_slots, int32_t* err_flag,
+                                      void* stream) {
+  if (batch < 0 || kmax < 1 || kmax > SEED_MAX_KMAX) return SEED_ERR_SHAPE;
+  if (batch == 0) return SEED_OK;
+  if (!tok || !parent || !n_nodes || !target_ids || !page_table || !ctx_lens || !accepted ||
+      !tokens || !path || !committed_slots || !err_flag)
+    return SEED_ERR_NULL;
+  if (max_pages <= 0 || page_size <= 0 || (long long)max_pages * page_size > INT32_MAX)
+    return SEED_ERR_RANGE;
+  return finish(seedk::launch_tree_accept(batch, kmax, tok, parent, n_nodes, target_ids,
+                                          page_table, max_pages, page_size, ctx_lens, accepted,
+                                          tokens, path, committed_slots, err_flag,
+                                          static_cast<cudaStream_t>(stream)));
+}
+
+seed_status_t seed_tree_kv_compact(const seed_cfg_t* cfg, int32_t batch, seed_kv_t kv,
+                                   const int32_t* path, const int32_t* accepted,
+                                   const int32_t* ctx_lens, int32_t* err_flag, void* stream) {
+  seed_status_t st = check_cfg(cfg);
+  if (st != SEED_OK) return st;
+  if (batch < 0) return SEED_ERR_SHAPE;
+  if (batch == 0) return SEED_OK;
+  if (!path || !accepted || !ctx_lens || !err_flag) return SEED_ERR_NULL;
+  if ((st = check_kv(kv)) != SEED_OK) return st;
+  if (misaligned16(kv.k) || misaligned16(kv.v)) return SEED_ERR_RANGE;
+  return finish(seedk::launch_tree_compact(
+      batch, cfg->hkv, cfg->head_dim, cfg->kmax, static_cast<uint16_t*>(kv.k),
+      static_cast<uint16_t*>(kv.v), kv.page_table, kv.max_pages, kv.num_pages, path, accepted,
+      ctx_lens, err_flag, static_cast<cudaStream_t>(stream)));
 }
 
 }  // extern "C"

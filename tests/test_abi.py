@@ -44,7 +44,7 @@ def test_exports_every_declared_function(lib):
 
 
 def test_version_and_strings(lib):
-    assert lib.seed_abi_version() == 1
+    assert lib.seed_abi_version() == 2
     for s in range(7):
         assert len(lib.seed_status_string(s)) > 0
     assert lib.seed_status_string(99) == b"unknown status"
@@ -58,7 +58,7 @@ def cfg(**kw):
 
 @pytest.mark.parametrize("kw,expect", [
     (dict(), OK), (dict(head_dim=96), ERR_UNSUP), (dict(hq=24, hkv=8), ERR_UNSUP),
-    (dict(hq=30, hkv=8), ERR_SHAPE), (dict(kmax=0), ERR_SHAPE), (dict(kmax=17), ERR_SHAPE),
+    (dict(hq=30, hkv=8), ERR_SHAPE), (dict(kmax=0), ERR_SHAPE), (dict(kmax=32), ERR_SHAPE), (dict(kmax=31), OK),
     (dict(page_size=32), ERR_UNSUP), (dict(scale=-1.0), ERR_SHAPE), (dict(head_dim=64), OK),
 ])
 def test_workspace_bytes_validates_cfg(lib, kw, expect):
@@ -127,8 +127,33 @@ def test_accept_host_checks(lib):
     args = [FAKE] * 4 + [8, 16] + [FAKE] * 5
     assert lib.seed_accept_commit(0, 4, *args, None) == OK
     assert lib.seed_accept_commit(2, 0, *args, None) == ERR_SHAPE
-    assert lib.seed_accept_commit(2, 17, *args, None) == ERR_SHAPE
+    assert lib.seed_accept_commit(2, 32, *args, None) == ERR_SHAPE
     bad = [FAKE, None] + args[2:]
     assert lib.seed_accept_commit(2, 4, *bad, None) == ERR_NULL
     bad = args[:4] + [0, 16] + args[6:]
     assert lib.seed_accept_commit(2, 4, *bad, None) == ERR_RANGE
+
+
+def test_tree_host_checks(lib):
+    c = cfg()
+    def tv(cf, B=2, q=FAKE, anc=FAKE, ws_bytes=1 << 30):
+        return lib.seed_tree_verify_attn(ctypes.byref(cf), B, q, FAKE, anc, kv(), FAKE, FAKE,
+                                         None, FAKE, ws_bytes, FAKE, None)
+    assert tv(c, B=0) == OK
+    assert tv(c, anc=None) == ERR_NULL
+    assert tv(c, q=None) == ERR_NULL
+    assert tv(c, ws_bytes=64) == ERR_WS
+    assert tv(cfg(head_dim=64)) == ERR_UNSUP              # tensor-core path only
+    assert tv(cfg(hq=64, hkv=8, kmax=16)) == ERR_UNSUP     # 8 * 17 rows > one 128-row tile
+    args = [FAKE] * 5 + [8, 16] + [FAKE] * 6
+    assert lib.seed_tree_accept_commit(0, 4, *args, None) == OK
+    assert lib.seed_tree_accept_commit(2, 32, *args, None) == ERR_SHAPE
+    bad = [FAKE, FAKE, None] + args[3:]
+    assert lib.seed_tree_accept_commit(2, 4, *bad, None) == ERR_NULL
+    bad = args[:5] + [0, 16] + args[7:]
+    assert lib.seed_tree_accept_commit(2, 4, *bad, None) == ERR_RANGE
+    assert lib.seed_tree_kv_compact(ctypes.byref(c), 0, kv(), FAKE, FAKE, FAKE, FAKE, None) == OK
+    assert lib.seed_tree_kv_compact(ctypes.byref(c), 2, kv(), None, FAKE, FAKE, FAKE,
+                                    None) == ERR_NULL
+    assert lib.seed_tree_kv_compact(ctypes.byref(c), 2, kv(num_pages=0), FAKE, FAKE, FAKE, FAKE,
+                                    None) == ERR_RANGE
