@@ -357,11 +357,13 @@ def attn_kernel_name(wl) -> str:
 
 
 def run_profile(args):
-    """--profile draft|verify: the appends of round 0 on the workload's two
+    """--profile draft|verify|tree: the appends of round 0 on the workload's two
     decoder layers, then `--reps` launches of one attention kind alternating
-    between them (a few hundred MB of KV, above the L2 size).  For ncu captures
-    of one launch (`-k regex:<kernel> -s 2 -c 1`); prints the algorithmic bytes
-    of each launch, no bench value."""
+    between them (a few hundred MB of KV, above the L2 size).  `tree` verifies
+    a full draft tree of kmax+1 nodes per sequence (binary, node i's parent is
+    (i-1)/2) with the tree mask of Sec. D.1.  For ncu captures of one launch
+    (`-k regex:<kernel> -s 2 -c 1`); prints the algorithmic bytes of each
+    launch, no bench value."""
     import torch
 
     from paper_2609_36590_gb300 import build
@@ -376,12 +378,27 @@ def run_profile(args):
     k_b = ins["k_b_np"]
     lens = dw.lens0
     dec = list(wl.dec_layers)
+    W = wl.kmax + 1
+    n_q = ins["n_q"]
+    if args.profile == "tree":
+        k_b = np.full(wl.batch, W - 1, dtype=np.int64)
+        n_q = torch.full((wl.batch,), W, dtype=torch.int32, device="cuda:0")
+        anc = np.zeros(W, dtype=np.int64)
+        for i in range(W):
+            a = i
+            while True:
+                anc[i] |= 1 << a
+                if a == 0:
+                    break
+                a = (a - 1) // 2
+        anc_dev = torch.from_numpy(np.tile(anc.astype(np.uint32).view(np.int32),
+                                           (wl.batch, 1))).to("cuda:0")
     for l in dec:
         q, kn, vn = ins["draft"][(1, l)]
         seed.seed_draft_kv_append(dw.cfg, kn, vn, ins["draft_lens"][0], dw.draft_k[l],
                                   dw.draft_v[l], dw.err)
         _, kn, vn = ins["verify"][l]
-        seed.seed_kv_append(dw.cfg, dw.kv[l], kn, vn, ins["n_q"], dw.ctx_lens, dw.err)
+        seed.seed_kv_append(dw.cfg, dw.kv[l], kn, vn, n_q, dw.ctx_lens, dw.err)
     torch.cuda.synchronize()
     ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.reps + 1)]
     ev[0].record()
@@ -389,13 +406,16 @@ def run_profile(args):
         l = dec[r % len(dec)]
         if args.profile == "draft":
             dw.draft_attn(ins, 1, l)
+        elif args.profile == "tree":
+            seed.seed_tree_verify_attn(dw.cfg, ins["verify"][l][0], n_q, anc_dev, dw.kv[l],
+                                       dw.ctx_lens, dw.out_v, dw.lse_v, dw.ws, dw.err)
         else:
             dw.verify_attn(ins, l)
         ev[r + 1].record()
     torch.cuda.synchronize()
     assert int(dw.err.item()) == 0, "device error flag raised"
     key = (1, dec[0]) if args.profile == "draft" else dec[0]
-    nbytes = attn_call_bytes(wl, args.profile, key, lens, k_b)
+    nbytes = attn_call_bytes(wl, "draft" if args.profile == "draft" else "verify", key, lens, k_b)
     print(json.dumps({"profile": args.profile, "workload": wl.name,
                       "kernel": attn_kernel_name(wl),
                       "sources": kernel_source_hash(attn_kernel_name(wl)),
@@ -521,7 +541,7 @@ def main():
     ap.add_argument("--impl", default="seed", choices=["seed", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=12.0)
-    ap.add_argument("--profile", choices=["draft", "verify"], default=None,
+    ap.add_argument("--profile", choices=["draft", "verify", "tree"], default=None,
                     help="launch one attention kind a few times for an ncu capture")
     ap.add_argument("--reps", type=int, default=3)
     args = ap.parse_args()
