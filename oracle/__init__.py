@@ -16,6 +16,9 @@ the paper (SEED: Self-Speculative Decoding via Implicit Encoder-Decoder):
   candidate sees the verified prefix and its own ancestral path), the greedy
   walk from the root with its bonus token, and the compaction of the accepted
   path's cache rows.
+* ``drafting``   -- confidence-aware dynamic drafting (Sec. D.1): the
+  drafter's distribution over the vocabulary, its top tokens, the
+  sibling-count rule on the top-1 probability and the stop threshold.
 * ``toy_model``  -- a tiny float64 transformer running Alg. 2 end to end (with
   a linear draft or a draft tree) and plain greedy decoding, for the
   exactness property of Sec. 4.1.

@@ -184,7 +184,8 @@ def seed_greedy(model: ToyLM, prompt, n_new: int, d: int, drafter: str = "model"
 
 def seed_tree_greedy(model: ToyLM, prompt, n_new: int, depth: int, width: int,
                      drafter: str = "model", reference=None, page_size: int = 4,
-                     page_seed: int = 0, mistake: str | None = None):
+                     page_seed: int = 0, mistake: str | None = None, tau: float | None = None,
+                     max_nodes: int = 32):
     """SEED with a draft tree and tree-based verification (Sec. D.1).
 
     Each round drafts a main branch of `depth` tokens with f_dec (as in Alg. 2);
@@ -197,13 +198,20 @@ def seed_tree_greedy(model: ToyLM, prompt, n_new: int, depth: int, width: int,
 
     mistake (planted, for the tests): 'causal' lets every node see all earlier
     packed rows (siblings included); 'nocompact' skips moving the accepted
-    rows.  Returns (tokens, accepted count per round).
+    rows.
+
+    tau (dynamic drafting, Sec. D.1): when given, `width` is ignored; each
+    step adds k children by the sibling-count rule on the drafter's top-1
+    probability p0, drafting stops after a step with p0 <= tau or at `depth`
+    steps, and the tree holds at most `max_nodes` nodes.  Returns (tokens,
+    accepted count per round).
     """
+    from . import drafting as _drafting
     from . import tree as _tree
 
     L = len(prompt) - 1
     pending = int(prompt[-1])
-    n_nodes = 1 + depth * width
+    n_nodes = 1 + depth * width if tau is None else max_nodes
     cap = len(prompt) + n_new + n_nodes + 2
     n_pages = -(-cap // page_size)
     pt = np.random.default_rng(page_seed).permutation(n_pages).astype(np.int32)
@@ -234,7 +242,12 @@ def seed_tree_greedy(model: ToyLM, prompt, n_new: int, depth: int, width: int,
                     q[0], _cache.gather_rows(kc[l], pt, L), _cache.gather_rows(vc[l], pt, L),
                     np.stack(dk[l]), np.stack(dv[l]), model.scale)
                 h = model.post(l, h, o[None])
-            order = [int(t) for t in np.argsort(-model.logits(h)[0], kind="stable")]
+            lg = model.logits(h)[0]
+            order = [int(t) for t in np.argsort(-lg, kind="stable")]
+            if tau is not None:
+                e = np.exp(lg - lg.max())
+                p0 = float(e.max() / e.sum())
+                width = min(int(_drafting.sibling_count([p0])[0]), max_nodes - len(tok))
             ref_i = len(out) + i - 1
             first = None
             if drafter == "perfect" and reference is not None and ref_i < len(reference):
@@ -248,6 +261,8 @@ def seed_tree_greedy(model: ToyLM, prompt, n_new: int, depth: int, width: int,
                 tok.append(t)
                 parent.append(main)
             main = base
+            if tau is not None and (p0 <= tau or len(tok) >= max_nodes):
+                break
         n = len(tok)
 
         # ---- verification: all nodes in one pass with the tree mask

@@ -220,3 +220,16 @@ def test_planted_tree_mistakes_are_noticed(model_and_ref, mistake):
                              mistake=mistake)[0]
             for depth in (2, 4) for dr in ("model", "adversarial")]
     assert any(o != ref for o in outs)
+
+
+@pytest.mark.parametrize("tau", [0.0, 0.5, 0.7, 1.01])
+def test_dynamic_drafting_trees_keep_greedy_ar(model_and_ref, tau):
+    """Trees built by the dynamic-drafting rule (k siblings from the drafter's
+    p0, stop after a step with p0 <= tau) and checked by tree verification
+    still emit exactly the greedy AR stream."""
+    m, ref = model_and_ref
+    out, rounds = seed_tree_greedy(m, PROMPT, N_NEW, 6, 1, tau=tau, max_nodes=24)
+    assert out == ref
+    assert all(0 <= n <= 6 for n in rounds)
+    if tau > 1.0:
+        assert all(n <= 1 for n in rounds)   # every step stops after its first level
