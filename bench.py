@@ -373,6 +373,9 @@ def run_profile(args):
 
     wl = WORKLOADS[args.workload]
     torch.cuda.set_device(0)
+    if args.profile == "head":
+        run_profile_head(args, wl)
+        return
     dw = DeviceWorkload(wl, device="cuda:0", layers=list(wl.dec_layers), rounds=2)
     ins = dw.round_inputs(0)
     k_b = ins["k_b_np"]
@@ -419,6 +422,45 @@ def run_profile(args):
     print(json.dumps({"profile": args.profile, "workload": wl.name,
                       "kernel": attn_kernel_name(wl),
                       "sources": kernel_source_hash(attn_kernel_name(wl)),
+                      "alg_bytes_per_launch": nbytes,
+                      "us": [round(ev[i].elapsed_time(ev[i + 1]) * 1e3, 1)
+                             for i in range(args.reps)]}))
+
+
+HEAD_D_MODEL, HEAD_VOCAB = 2560, 151936   # a 4B-scale (Qwen3-4B) LM head
+
+
+def run_profile_head(args, wl):
+    """--profile head: the dynamic-drafting head (LM head + softmax + top-10,
+    Sec. D.1) at 4B scale for the workload's batch, `--reps` launches.  The
+    head's 778 MB of weights are far above the L2 size.  Prints the
+    algorithmic bytes (weights once, plus h and the outputs) and the times."""
+    import torch
+
+    import paper_2609_36590_gb300 as seed
+
+    B, d, V = wl.batch, HEAD_D_MODEL, HEAD_VOCAB
+    g = torch.Generator(device="cuda:0").manual_seed(20260)
+    h = torch.randn(B, d, device="cuda:0", generator=g).to(torch.bfloat16)
+    w = (torch.randn(V, d, device="cuda:0", generator=g) / d ** 0.5).to(torch.bfloat16)
+    ids = torch.empty(B, 10, dtype=torch.int32, device="cuda:0")
+    probs = torch.empty(B, 10, device="cuda:0")
+    n_sib = torch.empty(B, dtype=torch.int32, device="cuda:0")
+    stop = torch.empty(B, dtype=torch.int32, device="cuda:0")
+    lse = torch.empty(B, device="cuda:0")
+    err = torch.zeros(1, dtype=torch.int32, device="cuda:0")
+    ws = seed.new_draft_head_workspace(B)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.reps + 1)]
+    torch.cuda.synchronize()
+    ev[0].record()
+    for r in range(args.reps):
+        seed.seed_draft_head_topk(h, w, 0.7, ids, probs, n_sib, stop, lse, ws, err)
+        ev[r + 1].record()
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0, "device error flag raised"
+    nbytes = V * d * 2 + B * d * 2 + B * (10 * 8 + 12)
+    print(json.dumps({"profile": "head", "workload": wl.name, "batch": B, "d_model": d,
+                      "vocab": V, "kernel": "head_tc_kernel",
                       "alg_bytes_per_launch": nbytes,
                       "us": [round(ev[i].elapsed_time(ev[i + 1]) * 1e3, 1)
                              for i in range(args.reps)]}))
@@ -541,7 +583,7 @@ def main():
     ap.add_argument("--impl", default="seed", choices=["seed", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=12.0)
-    ap.add_argument("--profile", choices=["draft", "verify", "tree"], default=None,
+    ap.add_argument("--profile", choices=["draft", "verify", "tree", "head"], default=None,
                     help="launch one attention kind a few times for an ncu capture")
     ap.add_argument("--reps", type=int, default=3)
     args = ap.parse_args()

@@ -264,6 +264,43 @@ seed_status_t seed_tree_kv_compact(const seed_cfg_t* cfg, int32_t batch, seed_kv
                                    const int32_t* ctx_lens, int32_t* err_flag, void* stream);
 
 /* ------------------------------------------------------------------------
+ * Confidence-aware dynamic drafting (Sec. D.1).  After each draft step the
+ * drafter's LM head gives a distribution p = softmax(W_out h) over the
+ * vocabulary.  Its top-1 probability p0 sets how many sibling candidates the
+ * tree gets at this step,
+ *     k = 1 if p0 > 0.95, 3 if 0.8 < p0 <= 0.95, 5 if 0.5 < p0 <= 0.8, else 10,
+ * and drafting goes on after a step only while p0 > tau (the step that falls
+ * to p0 <= tau still adds its k candidates).
+ * ------------------------------------------------------------------------ */
+#define SEED_DRAFT_TOPK 10             /* candidates returned per sequence */
+#define SEED_DRAFT_HEAD_MAX_BATCH 128  /* sequences per call */
+
+/* Bytes of workspace seed_draft_head_topk needs for `batch` sequences (no
+ * zeroing needed); 0 for a batch outside [1, SEED_DRAFT_HEAD_MAX_BATCH]. */
+size_t seed_draft_head_workspace_bytes(int32_t batch);
+
+/* The drafter's LM head with a fused softmax: for each sequence b, logits
+ * z = W_out h[b] (no bias, no temperature) over the whole vocabulary, never
+ * written out.
+ *   h          bf16 [batch, d_model]: the drafter's final hidden states (after
+ *              its output norm); d_model a multiple of 64
+ *   w_out      bf16 [vocab, d_model]: the LM head, row v = token v
+ *   tau        stop threshold
+ *   ids        int32 [batch, 10]: the 10 most probable tokens, decreasing
+ *              probability, equal logits in increasing id order
+ *   probs      f32 [batch, 10]: their probabilities (probs[b, 0] = p0)
+ *   n_sib      int32 [batch]: k by the rule above
+ *   stop       int32 [batch]: 1 when p0 <= tau
+ *   lse        f32 [batch]: natural log of sum_v exp(z_v), or NULL
+ * Runs on the tensor cores (bf16 inputs, f32 accumulation).  batch <= 128,
+ * vocab >= 10.  Device errors: SEED_DEVERR_TIMEOUT only. */
+seed_status_t seed_draft_head_topk(int32_t batch, int32_t d_model, int32_t vocab,
+                                   const void* h, const void* w_out, float tau,
+                                   int32_t* ids, float* probs, int32_t* n_sib,
+                                   int32_t* stop, float* lse, void* ws, size_t ws_bytes,
+                                   int32_t* err_flag, void* stream);
+
+/* ------------------------------------------------------------------------
  * Library convenience with no counterpart in the paper: verify attention
  * without a caller-provided workspace.
  *

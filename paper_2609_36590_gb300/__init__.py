@@ -10,7 +10,8 @@ Entry points carry the C names: seed_workspace_bytes, seed_draft_kv_append,
 seed_draft_attn, seed_kv_append, seed_verify_attn, seed_accept_commit, and
 seed_verify_attn_noalloc (verify attention on the library's built-in scratch,
 for callers that cannot provide a workspace), and the tree-verification calls
-seed_tree_verify_attn, seed_tree_accept_commit, seed_tree_kv_compact.
+seed_tree_verify_attn, seed_tree_accept_commit, seed_tree_kv_compact, and the
+dynamic-drafting head seed_draft_head_topk.
 """
 
 from __future__ import annotations
@@ -62,6 +63,9 @@ _SIGS = {
     "seed_tree_accept_commit": (_I, [_I, _I, _P, _P, _P, _P, _P, _I, _I, _P, _P, _P, _P, _P,
                                      _P, _P]),
     "seed_tree_kv_compact": (_I, [ctypes.POINTER(_Cfg), _I, _KV, _P, _P, _P, _P, _P]),
+    "seed_draft_head_workspace_bytes": (ctypes.c_size_t, [_I]),
+    "seed_draft_head_topk": (_I, [_I, _I, _I, _P, _P, ctypes.c_float, _P, _P, _P, _P, _P, _P,
+                                  ctypes.c_size_t, _P, _P]),
 }
 
 
@@ -301,6 +305,32 @@ def seed_tree_kv_compact(cfg: SeedConfig, kv: PagedKV, path, accepted, ctx_lens,
         _t(path, torch.int32, (B, cfg.kmax + 1), "path"),
         _t(accepted, torch.int32, (B,), "accepted"),
         _t(ctx_lens, torch.int32, (B,), "ctx_lens"),
+        _t(err, torch.int32, (1,), "err"), _stream(stream)))
+
+
+def new_draft_head_workspace(batch: int, device=None) -> torch.Tensor:
+    n = _lib.seed_draft_head_workspace_bytes(batch)
+    if n == 0:
+        raise SeedError("batch outside the supported range")
+    return torch.empty(int(n), dtype=torch.uint8, device=device or "cuda")
+
+
+def seed_draft_head_topk(h, w_out, tau: float, ids, probs, n_sib, stop, lse, ws, err,
+                         stream=None) -> None:
+    """LM head + softmax + top-10 per sequence, sibling count and stop flag."""
+    B, d = h.shape
+    V = w_out.shape[0]
+    _check(_lib.seed_draft_head_topk(
+        B, d, V,
+        _t(h, torch.bfloat16, (B, d), "h"),
+        _t(w_out, torch.bfloat16, (V, d), "w_out"),
+        float(tau),
+        _t(ids, torch.int32, (B, 10), "ids"),
+        _t(probs, torch.float32, (B, 10), "probs"),
+        _t(n_sib, torch.int32, (B,), "n_sib"),
+        _t(stop, torch.int32, (B,), "stop"),
+        _t(lse, torch.float32, (B,), "lse") if lse is not None else None,
+        _t(ws, torch.uint8, None, "ws"), ws.numel(),
         _t(err, torch.int32, (1,), "err"), _stream(stream)))
 
 

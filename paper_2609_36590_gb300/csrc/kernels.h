@@ -101,6 +101,24 @@ cudaError_t launch_tree_compact(int32_t B, int32_t hkv, int32_t head_dim, int32_
 
 int device_sm_count();
 
+// Drafter LM head with fused softmax and top-10 (head_tc.cu).
+constexpr int kHeadMaxCtas = 256;
+struct HeadParams {
+  float* part;        // [ctas, B, 24] partial records
+  int32_t* ids;       // [B, 10]
+  float* probs;       // [B, 10]
+  int32_t* n_sib;     // [B]
+  int32_t* stop;      // [B]
+  float* lse;         // [B] or null
+  int32_t* err;
+  int32_t B, d, V;
+  float tau;
+};
+int head_ctas(int32_t vocab);
+size_t head_workspace_bytes(int32_t batch);
+cudaError_t launch_head(const HeadParams& p, const void* h, const void* w, int nctas,
+                        cudaStream_t st);
+
 // Tensor-core draft and verify attention (attn_tc.cu).
 constexpr int kTcMaxCtas = 256;     // most CTAs of one launch (two record slots each)
 

@@ -311,4 +311,38 @@ seed_status_t seed_tree_kv_compact(const seed_cfg_t* cfg, int32_t batch, seed_kv
       ctx_lens, err_flag, static_cast<cudaStream_t>(stream)));
 }
 
+size_t seed_draft_head_workspace_bytes(int32_t batch) {
+  if (batch < 1 || batch > SEED_DRAFT_HEAD_MAX_BATCH) return 0;
+  return seedk::head_workspace_bytes(batch);
+}
+
+seed_status_t seed_draft_head_topk(int32_t batch, int32_t d_model, int32_t vocab,
+                                   const void* h, const void* w_out, float tau, int32_t* ids,
+                                   float* probs, int32_t* n_sib, int32_t* stop, float* lse,
+                                   void* ws, size_t ws_bytes, int32_t* err_flag, void* stream) {
+  if (batch < 0 || batch > SEED_DRAFT_HEAD_MAX_BATCH) return SEED_ERR_SHAPE;
+  if (d_model <= 0 || d_model % 64 != 0 || vocab < SEED_DRAFT_TOPK) return SEED_ERR_SHAPE;
+  if (!(tau >= 0.f) || std::isinf(tau)) return SEED_ERR_SHAPE;
+  if (batch == 0) return SEED_OK;
+  if (!h || !w_out || !ids || !probs || !n_sib || !stop || !ws || !err_flag) return SEED_ERR_NULL;
+  if (misaligned16(h) || misaligned16(w_out)) return SEED_ERR_RANGE;
+  if ((reinterpret_cast<uintptr_t>(ws) & 15u) != 0 ||
+      ws_bytes < seedk::head_workspace_bytes(batch))
+    return SEED_ERR_WORKSPACE;
+  seedk::HeadParams p{};
+  p.part = static_cast<float*>(ws);
+  p.ids = ids;
+  p.probs = probs;
+  p.n_sib = n_sib;
+  p.stop = stop;
+  p.lse = lse;
+  p.err = err_flag;
+  p.B = batch;
+  p.d = d_model;
+  p.V = vocab;
+  p.tau = tau;
+  return finish(seedk::launch_head(p, h, w_out, seedk::head_ctas(vocab),
+                                   static_cast<cudaStream_t>(stream)));
+}
+
 }  // extern "C"

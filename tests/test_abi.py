@@ -157,3 +157,21 @@ def test_tree_host_checks(lib):
                                     None) == ERR_NULL
     assert lib.seed_tree_kv_compact(ctypes.byref(c), 2, kv(num_pages=0), FAKE, FAKE, FAKE, FAKE,
                                     None) == ERR_RANGE
+
+
+def test_draft_head_host_checks(lib):
+    args = [FAKE] * 4 + [None, FAKE, 1 << 30, FAKE, None]   # ids..stop, lse, ws, bytes, err, stream
+    def call(B=4, d=256, V=1000, h=FAKE, tau=0.7, a=None):
+        return lib.seed_draft_head_topk(B, d, V, h, FAKE, ctypes.c_float(tau), *(a or args))
+    assert call(B=0) == OK
+    assert call(B=129) == ERR_SHAPE
+    assert call(d=100) == ERR_SHAPE
+    assert call(V=5) == ERR_SHAPE
+    assert call(tau=-1.0) == ERR_SHAPE
+    assert call(h=None) == ERR_NULL
+    assert call(h=FAKE + 8) == ERR_RANGE
+    small = args[:6] + [64] + args[7:]
+    assert call(a=small) == ERR_WS
+    assert lib.seed_draft_head_workspace_bytes(0) == 0
+    assert lib.seed_draft_head_workspace_bytes(129) == 0
+    assert lib.seed_draft_head_workspace_bytes(64) > 0
