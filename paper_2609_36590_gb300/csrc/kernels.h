@@ -104,7 +104,7 @@ int device_sm_count();
 // Drafter LM head with fused softmax and top-10 (head_tc.cu).
 constexpr int kHeadMaxCtas = 256;
 struct HeadParams {
-  float* part;        // [ctas, B, 24] partial records
+  float* part;        // [ctas * 4, B, 24] partial records
   int32_t* ids;       // [B, 10]
   float* probs;       // [B, 10]
   int32_t* n_sib;     // [B]
