@@ -19,6 +19,11 @@ the paper (SEED: Self-Speculative Decoding via Implicit Encoder-Decoder):
 * ``drafting``   -- confidence-aware dynamic drafting (Sec. D.1): the
   drafter's distribution over the vocabulary, its top tokens, the
   sibling-count rule on the top-1 probability and the stop threshold.
+* ``draft_step`` -- one whole draft step (Sec. 4.1 drafting; the work the
+  computational-cost appendix counts): raw embedding, the decoder layers in
+  the pre-norm form of the paper's Qwen3 models (RMS norms, q/k norms, RoPE,
+  grouped attention over the deep cache plus the draft rows, SwiGLU MLP),
+  final norm and the dynamic-drafting head.
 * ``toy_model``  -- a tiny float64 transformer running Alg. 2 end to end (with
   a linear draft or a draft tree) and plain greedy decoding, for the
   exactness property of Sec. 4.1.
