@@ -45,7 +45,7 @@
 extern "C" {
 #endif
 
-#define SEED_ABI_VERSION 2
+#define SEED_ABI_VERSION 3
 #define SEED_MAX_KMAX 31        /* largest supported draft length d (32 rows per sequence) */
 
 typedef enum {
@@ -68,6 +68,7 @@ typedef enum {
 #define SEED_DEVERR_WORKSPACE 32  /* more work units than the workspace holds       */
 #define SEED_DEVERR_TIMEOUT   64  /* a bounded on-chip wait gave up (never expected) */
 #define SEED_DEVERR_TREE      128 /* a draft tree's parents or accepted path are invalid */
+#define SEED_DEVERR_TOKEN     256 /* a token id outside [0, vocab)                      */
 
 /* Shapes of one model's attention.  Supported: head_dim in {64, 128};
  * hq / hkv in {1, 2, 4, 8}; page_size == 16; 1 <= kmax <= SEED_MAX_KMAX.
@@ -299,6 +300,101 @@ seed_status_t seed_draft_head_topk(int32_t batch, int32_t d_model, int32_t vocab
                                    int32_t* ids, float* probs, int32_t* n_sib,
                                    int32_t* stop, float* lse, void* ws, size_t ws_bytes,
                                    int32_t* err_flag, void* stream);
+
+/* ------------------------------------------------------------------------
+ * The whole draft step on the device (Sec. 4.1 "cheap drafting"; the work per
+ * draft token that the paper's computational-cost appendix counts: per
+ * decoder layer W_Q, W_K, W_V, W_O and three MLP matrices, then the head).
+ * The decoder layers are the model's last l - l' layers, in the pre-norm form
+ * of the paper's Qwen3 models:
+ *   a = RMSNorm(x; g_attn); q, k, v = a W_qkv^T (q heads, then k, then v);
+ *   q, k = RoPE(RMSNorm_head(q; g_q)), RoPE(RMSNorm_head(k; g_k));
+ *   (k, v) -> draft row i-1; o = draft attention; x += o W_o^T;
+ *   m = RMSNorm(x; g_mlp); x += (silu(m W_gate^T) * (m W_up^T)) W_down^T.
+ * The residual stream x is f32; the operands of every product (a, q, k, v,
+ * o, m and the MLP activation) are bf16.  RoPE pairs element i with i + D/2
+ * at angle pos * theta^(-2i/D), pos = ctx_len + draft_len - 1.
+ * Weights are bf16, row-major in nn.Linear layout [out, in], 16-byte aligned.
+ * ------------------------------------------------------------------------ */
+
+/* The three epilogues of seed_linear. */
+#define SEED_LINEAR_F32       0  /* y  = x W^T, f32 [batch, n_out]                   */
+#define SEED_LINEAR_RESID_F32 1  /* y += x W^T, f32 [batch, n_out] updated in place   */
+#define SEED_LINEAR_SWIGLU    2  /* y  = bf16(silu(x W^T) * (x W2^T)), bf16 [batch, n_out] */
+#define SEED_LINEAR_MAX_BATCH 128
+
+/* Workspace bytes of seed_linear for these sizes and epilogue on the current
+ * device: a fixed block of per-tile arrival counters, then stream-K partial
+ * sums.  It must be 256-byte aligned and ZERO-FILLED before its first use;
+ * every call leaves the counters zero again, so one workspace (of the largest
+ * size needed) serves any sequence of calls on one stream.  0 for sizes
+ * seed_linear rejects. */
+size_t seed_linear_workspace_bytes(int32_t batch, int32_t n_out, int32_t k_in, int32_t epilogue);
+
+/* y (epilogue) x W^T on the tensor cores, one pass over W.
+ *   x      bf16 [batch, k_in], batch in [1, SEED_LINEAR_MAX_BATCH], k_in % 64 == 0,
+ *          n_out <= 524288
+ *   w      bf16 [n_out, k_in]; w2 bf16 [n_out, k_in] for SEED_LINEAR_SWIGLU
+ *          (the up projection, w being the gate), else NULL
+ *   y      see the epilogue; never aliases x
+ * Errors: SEED_ERR_SHAPE (sizes, epilogue), SEED_ERR_NULL, SEED_ERR_RANGE
+ * (a pointer not 16-byte aligned), SEED_ERR_WORKSPACE.  batch 0 is a no-op.
+ * Device errors: SEED_DEVERR_TIMEOUT only. */
+seed_status_t seed_linear(int32_t batch, int32_t k_in, int32_t n_out, const void* x,
+                          const void* w, const void* w2, int32_t epilogue, void* y,
+                          void* ws, size_t ws_bytes, int32_t* err_flag, void* stream);
+
+/* x[b] = W_emb[tokens[b]] as f32 [batch, d_model] (the raw embedding H^0 the
+ * drafter is fed, Sec. 4.1).  W_emb bf16 [vocab, d_model].
+ * Device errors: SEED_DEVERR_TOKEN (that row is left untouched). */
+seed_status_t seed_embed(int32_t batch, int32_t d_model, int32_t vocab, const int32_t* tokens,
+                         const void* w_emb, float* x, int32_t* err_flag, void* stream);
+
+/* y = bf16(x / sqrt(mean(x^2) + eps) * gamma) row by row; x f32 [rows, n],
+ * gamma bf16 [n], y bf16 [rows, n]. */
+seed_status_t seed_rmsnorm(int32_t rows, int32_t n, const float* x, const void* gamma,
+                           float eps, void* y, void* stream);
+
+/* One decoder layer's weights (all bf16, nn.Linear layout). */
+typedef struct {
+  int32_t d_model;       /* multiple of 64 */
+  int32_t d_ff;          /* multiple of 64 */
+  float rms_eps;         /* e.g. 1e-6 */
+  float rope_theta;      /* e.g. 1e6 */
+  const void* g_attn;    /* [d_model] */
+  const void* w_qkv;     /* [(hq + 2 hkv) head_dim, d_model] */
+  const void* g_q;       /* [head_dim] */
+  const void* g_k;       /* [head_dim] */
+  const void* w_o;       /* [d_model, hq head_dim] */
+  const void* g_mlp;     /* [d_model] */
+  const void* w_gate;    /* [d_ff, d_model] */
+  const void* w_up;      /* [d_ff, d_model] */
+  const void* w_down;    /* [d_model, d_ff] */
+} seed_decoder_layer_t;
+
+/* Workspace bytes of seed_draft_layer (256-byte aligned, ZERO-FILLED before
+ * its first use; every call leaves its counters zeroed again). */
+size_t seed_draft_layer_workspace_bytes(const seed_cfg_t* cfg, const seed_decoder_layer_t* layer,
+                                        int32_t batch);
+
+/* One decoder layer of draft step i for a batch (head_dim 64 or 128):
+ *   x          f32 [batch, d_model], the residual stream, updated in place
+ *   ctx_kv     this layer's committed cache (the deep KV, read only)
+ *   ctx_lens   int32 [batch] committed rows L
+ *   draft_k/v  this layer's draft scratch; row i-1 is written
+ *   draft_lens int32 [batch]: i after this step (1..kmax); 0 skips the
+ *              sequence (its x row is then unspecified)
+ * The step's token sits at position L + i - 1.  Launches norm, QKV product,
+ * q/k norm + RoPE, draft KV append, draft attention, output product with
+ * residual, norm, gate/up product with SwiGLU and down product with residual,
+ * in this order on `stream`.
+ * Errors: as seed_draft_attn and seed_linear.  Device errors: as
+ * seed_draft_attn, plus SEED_DEVERR_TIMEOUT. */
+seed_status_t seed_draft_layer(const seed_cfg_t* cfg, int32_t batch,
+                               const seed_decoder_layer_t* layer, float* x, seed_kv_t ctx_kv,
+                               const int32_t* ctx_lens, void* draft_k, void* draft_v,
+                               const int32_t* draft_lens, void* ws, size_t ws_bytes,
+                               int32_t* err_flag, void* stream);
 
 /* ------------------------------------------------------------------------
  * Library convenience with no counterpart in the paper: verify attention

@@ -10,8 +10,9 @@ Entry points carry the C names: seed_workspace_bytes, seed_draft_kv_append,
 seed_draft_attn, seed_kv_append, seed_verify_attn, seed_accept_commit, and
 seed_verify_attn_noalloc (verify attention on the library's built-in scratch,
 for callers that cannot provide a workspace), and the tree-verification calls
-seed_tree_verify_attn, seed_tree_accept_commit, seed_tree_kv_compact, and the
-dynamic-drafting head seed_draft_head_topk.
+seed_tree_verify_attn, seed_tree_accept_commit, seed_tree_kv_compact, the
+dynamic-drafting head seed_draft_head_topk, and the draft step on the device:
+seed_linear, seed_embed, seed_rmsnorm and seed_draft_layer.
 """
 
 from __future__ import annotations
@@ -29,13 +30,20 @@ SEED_OK = 0
 SEED_ERR_SCRATCH_LIMIT = 7
 NOALLOC_SCRATCH_BYTES = 32 << 20   # SEED_NOALLOC_SCRATCH_BYTES of seed.h
 DEVERR = {1: "ctx_len", 2: "draft_len", 4: "n_q", 8: "page", 16: "k_b", 32: "workspace",
-          64: "timeout", 128: "tree"}
+          64: "timeout", 128: "tree", 256: "token"}
 MAX_KMAX = 31
 
 
 class _Cfg(ctypes.Structure):
     _fields_ = [("hq", ctypes.c_int32), ("hkv", ctypes.c_int32), ("head_dim", ctypes.c_int32),
                 ("page_size", ctypes.c_int32), ("kmax", ctypes.c_int32), ("scale", ctypes.c_float)]
+
+
+class _Layer(ctypes.Structure):
+    _fields_ = [("d_model", ctypes.c_int32), ("d_ff", ctypes.c_int32),
+                ("rms_eps", ctypes.c_float), ("rope_theta", ctypes.c_float)] + [
+        (n, ctypes.c_void_p) for n in ("g_attn", "w_qkv", "g_q", "g_k", "w_o", "g_mlp", "w_gate",
+                                       "w_up", "w_down")]
 
 
 class _KV(ctypes.Structure):
@@ -64,6 +72,14 @@ _SIGS = {
                                      _P, _P]),
     "seed_tree_kv_compact": (_I, [ctypes.POINTER(_Cfg), _I, _KV, _P, _P, _P, _P, _P]),
     "seed_draft_head_workspace_bytes": (ctypes.c_size_t, [_I]),
+    "seed_linear_workspace_bytes": (ctypes.c_size_t, [_I, _I, _I, _I]),
+    "seed_linear": (_I, [_I, _I, _I, _P, _P, _P, _I, _P, _P, ctypes.c_size_t, _P, _P]),
+    "seed_embed": (_I, [_I, _I, _I, _P, _P, _P, _P, _P]),
+    "seed_rmsnorm": (_I, [_I, _I, _P, _P, ctypes.c_float, _P, _P]),
+    "seed_draft_layer_workspace_bytes": (ctypes.c_size_t, [ctypes.POINTER(_Cfg),
+                                                           ctypes.POINTER(_Layer), _I]),
+    "seed_draft_layer": (_I, [ctypes.POINTER(_Cfg), _I, ctypes.POINTER(_Layer), _P, _KV, _P, _P,
+                              _P, _P, _P, ctypes.c_size_t, _P, _P]),
     "seed_draft_head_topk": (_I, [_I, _I, _I, _P, _P, ctypes.c_float, _P, _P, _P, _P, _P, _P,
                                   ctypes.c_size_t, _P, _P]),
 }
@@ -349,6 +365,93 @@ def seed_accept_commit(kmax: int, draft_ids, target_ids, k_b, page_table, page_s
         _t(tokens, torch.int32, (B, kmax + 1), "tokens"),
         _t(committed_slots, torch.int32, (B, kmax + 1), "committed_slots"),
         _t(err, torch.int32, (1,), "err"), _stream(stream)))
+
+
+LINEAR_F32, LINEAR_RESID_F32, LINEAR_SWIGLU = 0, 1, 2
+
+
+def new_linear_workspace(batch: int, n_out: int, k_in: int, epilogue: int,
+                         device=None) -> torch.Tensor:
+    """A zero-filled workspace for seed_linear with these sizes."""
+    n = _lib.seed_linear_workspace_bytes(batch, n_out, k_in, epilogue)
+    if n == 0:
+        raise SeedError("invalid seed_linear sizes")
+    return torch.zeros(int(n), dtype=torch.uint8, device=device or "cuda")
+
+
+def seed_linear(x, w, y, ws, err, epilogue: int = LINEAR_F32, w2=None, stream=None) -> None:
+    """y (epilogue) x w^T: x bf16 [B, K], w (and w2 for SwiGLU) bf16 [N, K];
+    y f32 [B, N] (F32, RESID_F32) or bf16 [B, N] (SWIGLU)."""
+    B, K = x.shape
+    N = w.shape[0]
+    ydt = torch.bfloat16 if epilogue == LINEAR_SWIGLU else torch.float32
+    _check(_lib.seed_linear(
+        B, K, N, _t(x, torch.bfloat16, (B, K), "x"), _t(w, torch.bfloat16, (N, K), "w"),
+        _t(w2, torch.bfloat16, (N, K), "w2") if w2 is not None else None, epilogue,
+        _t(y, ydt, (B, N), "y"), _t(ws, torch.uint8, None, "ws"), ws.numel(),
+        _t(err, torch.int32, (1,), "err"), _stream(stream)))
+
+
+def seed_embed(tokens, w_emb, x, err, stream=None) -> None:
+    B = tokens.shape[0]
+    V, d = w_emb.shape
+    _check(_lib.seed_embed(B, d, V, _t(tokens, torch.int32, (B,), "tokens"),
+                           _t(w_emb, torch.bfloat16, (V, d), "w_emb"),
+                           _t(x, torch.float32, (B, d), "x"), _t(err, torch.int32, (1,), "err"),
+                           _stream(stream)))
+
+
+def seed_rmsnorm(x, gamma, eps: float, y, stream=None) -> None:
+    rows, n = x.shape
+    _check(_lib.seed_rmsnorm(rows, n, _t(x, torch.float32, (rows, n), "x"),
+                             _t(gamma, torch.bfloat16, (n,), "gamma"), eps,
+                             _t(y, torch.bfloat16, (rows, n), "y"), _stream(stream)))
+
+
+@dataclass
+class DecoderLayer:
+    """One decoder layer's bf16 weights (nn.Linear layout) for seed_draft_layer."""
+    g_attn: torch.Tensor
+    w_qkv: torch.Tensor
+    g_q: torch.Tensor
+    g_k: torch.Tensor
+    w_o: torch.Tensor
+    g_mlp: torch.Tensor
+    w_gate: torch.Tensor
+    w_up: torch.Tensor
+    w_down: torch.Tensor
+    rms_eps: float = 1e-6
+    rope_theta: float = 1e6
+
+    def c(self, cfg: SeedConfig) -> _Layer:
+        dm, F = self.w_gate.shape[1], self.w_gate.shape[0]
+        D, nqkv = cfg.head_dim, (cfg.hq + 2 * cfg.hkv) * cfg.head_dim
+        shapes = dict(g_attn=(dm,), w_qkv=(nqkv, dm), g_q=(D,), g_k=(D,), w_o=(dm, cfg.hq * D),
+                      g_mlp=(dm,), w_gate=(F, dm), w_up=(F, dm), w_down=(dm, F))
+        ptr = {n: _t(getattr(self, n), torch.bfloat16, shp, n) for n, shp in shapes.items()}
+        return _Layer(dm, F, self.rms_eps, self.rope_theta, *[ptr[n] for n in shapes])
+
+
+def new_draft_layer_workspace(cfg: SeedConfig, layer: DecoderLayer, batch: int,
+                              device=None) -> torch.Tensor:
+    c, lc = cfg.c(), layer.c(cfg)
+    n = _lib.seed_draft_layer_workspace_bytes(ctypes.byref(c), ctypes.byref(lc), batch)
+    if n == 0:
+        raise SeedError("invalid seed_draft_layer configuration")
+    return torch.zeros(int(n), dtype=torch.uint8, device=device or "cuda")
+
+
+def seed_draft_layer(cfg: SeedConfig, layer: DecoderLayer, x, ctx_kv: PagedKV, ctx_lens, draft_k,
+                     draft_v, draft_lens, ws, err, stream=None) -> None:
+    B, dm = x.shape
+    c, lc = cfg.c(), layer.c(cfg)
+    _check(_lib.seed_draft_layer(
+        ctypes.byref(c), B, ctypes.byref(lc), _t(x, torch.float32, (B, dm), "x"),
+        _kv_checked(cfg, ctx_kv, B), _t(ctx_lens, torch.int32, (B,), "ctx_lens"),
+        _t(draft_k, torch.bfloat16, (B, cfg.hkv, cfg.kmax, cfg.head_dim), "draft_k"),
+        _t(draft_v, torch.bfloat16, (B, cfg.hkv, cfg.kmax, cfg.head_dim), "draft_v"),
+        _t(draft_lens, torch.int32, (B,), "draft_lens"), _t(ws, torch.uint8, None, "ws"),
+        ws.numel(), _t(err, torch.int32, (1,), "err"), _stream(stream)))
 
 
 def library() -> ctypes.CDLL:

@@ -119,6 +119,34 @@ size_t head_workspace_bytes(int32_t batch);
 cudaError_t launch_head(const HeadParams& p, const void* h, const void* w, int nctas,
                         cudaStream_t st);
 
+// Skinny GEMM for the drafter's decoder layers (linear_tc.cu).
+constexpr int kLinearMaxCtas = 256;
+constexpr int kLinearMaxTiles = 4096;                  // n_out <= 4096 * 128
+constexpr size_t kLinearCntBytes = kLinearMaxTiles * sizeof(int32_t);
+enum LinearEpi : int32_t { kEpiF32 = 0, kEpiResidF32 = 1, kEpiSwigluBf16 = 2 };
+struct LinearParams {
+  void* y;            // f32 [B, N] (kEpiF32, kEpiResidF32) or bf16 [B, N] (kEpiSwigluBf16)
+  float* part;        // [ctas * 2, (1|2) * nb, 128] partial accumulators
+  int32_t* cnt;       // [kLinearMaxTiles] arrival counters, zero between calls
+  int32_t* err;
+  int32_t B, K, N, epi;
+};
+int linear_ctas(int32_t n_out, int32_t k_in);
+size_t linear_workspace_bytes(int32_t batch, int32_t n_out, int32_t k_in, int32_t epi);
+cudaError_t launch_linear(LinearParams p, const void* x, const void* w, const void* w2, void* ws,
+                          cudaStream_t st);
+
+// The small steps of a draft step (draft_ops.cu).
+cudaError_t launch_embed(int32_t B, int32_t d, int32_t vocab, const int32_t* tokens,
+                         const void* w, float* x, int32_t* err, cudaStream_t st);
+cudaError_t launch_rmsnorm(int32_t rows, int32_t n, const float* x, const void* gamma, float eps,
+                           void* y, cudaStream_t st);
+cudaError_t launch_qk_norm_rope(int32_t B, int32_t hq, int32_t hkv, int32_t D, const float* qkv,
+                                const void* gq, const void* gk, const int32_t* ctx_lens,
+                                const int32_t* draft_lens, float theta, float eps, void* q,
+                                void* k, void* v, cudaStream_t st);
+cudaError_t launch_f32_to_bf16(size_t n, const float* x, void* y, cudaStream_t st);
+
 // Tensor-core draft and verify attention (attn_tc.cu).
 constexpr int kTcMaxCtas = 256;     // most CTAs of one launch (two record slots each)
 

@@ -44,7 +44,7 @@ def test_exports_every_declared_function(lib):
 
 
 def test_version_and_strings(lib):
-    assert lib.seed_abi_version() == 2
+    assert lib.seed_abi_version() == 3
     for s in range(7):
         assert len(lib.seed_status_string(s)) > 0
     assert lib.seed_status_string(99) == b"unknown status"
@@ -175,3 +175,47 @@ def test_draft_head_host_checks(lib):
     assert lib.seed_draft_head_workspace_bytes(0) == 0
     assert lib.seed_draft_head_workspace_bytes(129) == 0
     assert lib.seed_draft_head_workspace_bytes(64) > 0
+
+
+def test_linear_host_checks(lib):
+    def call(B=4, K=256, N=300, x=FAKE, w=FAKE, w2=None, epi=0, y=FAKE, ws=FAKE, nbytes=1 << 30,
+             err=FAKE):
+        return lib.seed_linear(B, K, N, x, w, w2, epi, y, ws, nbytes, err, None)
+    assert call(B=0) == OK
+    assert call(B=129) == ERR_SHAPE
+    assert call(K=100) == ERR_SHAPE             # K not a multiple of 64
+    assert call(N=0) == ERR_SHAPE
+    assert call(epi=3) == ERR_SHAPE
+    assert call(x=None) == ERR_NULL
+    assert call(epi=2) == ERR_NULL              # SwiGLU needs the up projection
+    assert call(w=FAKE + 8) == ERR_RANGE
+    assert call(ws=FAKE + 128) == ERR_WS
+    assert call(nbytes=64) == ERR_WS
+    assert lib.seed_linear_workspace_bytes(4, 300, 100, 0) == 0
+    assert lib.seed_linear_workspace_bytes(0, 300, 256, 0) == 0
+    a = lib.seed_linear_workspace_bytes(16, 300, 256, 0)
+    assert 0 < a < lib.seed_linear_workspace_bytes(16, 300, 256, 2)
+
+
+def test_draft_layer_host_checks(lib):
+    c = _Cfg(32, 8, 128, 16, 8, 0.0)
+    P = [FAKE] * 9
+
+    def layer(dm=2560, F=9728, eps=1e-6, theta=1e6):
+        return seed._Layer(dm, F, eps, theta, *P)
+
+    def call(cf=c, B=2, L=None, x=FAKE, ws=FAKE, nbytes=1 << 34):
+        return lib.seed_draft_layer(ctypes.byref(cf), B, ctypes.byref(L or layer()), x, kv(), FAKE,
+                                    FAKE, FAKE, FAKE, ws, nbytes, FAKE, None)
+    assert call(B=0) == OK
+    assert call(B=129) == ERR_SHAPE
+    assert call(L=layer(dm=100)) == ERR_UNSUP
+    assert call(L=layer(theta=0.5)) == ERR_UNSUP
+    assert call(cf=_Cfg(32, 8, 96, 16, 8, 0.0)) == ERR_UNSUP
+    assert call(x=None) == ERR_NULL
+    assert call(x=FAKE + 4) == ERR_RANGE
+    assert call(nbytes=1024) == ERR_WS
+    assert call(ws=FAKE + 16) == ERR_WS
+    n = lib.seed_draft_layer_workspace_bytes(ctypes.byref(c), ctypes.byref(layer()), 4)
+    assert n > lib.seed_workspace_bytes(ctypes.byref(c), 4)
+    assert lib.seed_draft_layer_workspace_bytes(ctypes.byref(c), ctypes.byref(layer()), 0) == 0

@@ -1,0 +1,319 @@
+"""GPU parity of the draft step on the device (Sec. 4.1 drafting through the
+model's last layers) through the C ABI against the oracle:
+
+* seed_linear, all three epilogues, over shapes whose (tile, slab) units
+  split tiles across many CTAs (stream-K partials and last-arriver sums),
+  ragged row tiles and every batch class: within the float32-accumulation
+  bound of the exact float64 product (and half a bf16 step for SwiGLU);
+  deterministic, and the workspace counters are zero again afterwards;
+* seed_embed (exact) and seed_rmsnorm (within one bf16 step);
+* seed_draft_layer for head_dim 64 and 128 against the oracle's layer
+  (which rounds the same operands to bf16): the appended draft K/V rows and
+  the residual stream, including skipped sequences;
+* a whole 4B-sized draft step (two layers, final norm, dynamic-drafting head)
+  on sampled sequences.
+
+Tolerances: the device rounds the same operands to bf16 as the oracle but
+from float32 values, so an operand lands one bf16 step away where the exact
+value sits near a rounding boundary.  For the projections (K/V rows) that is
+rare: they differ from the oracle's in at most 1 % of elements, by one step.
+The attention output carries the attention tolerance (2e-3 absolute, about
+0.25 % of |o|), and rounding it to bf16 then moves about half of its elements
+by one step (0.4 %); summed through W_o with random signs that stays near
+0.5 % of the update.  The residual stream is therefore checked to 5e-3 of its
+scale (max abs over the rows), and the final norm's output to 1e-2."""
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import draft_step as DS
+from oracle import drafting as OD
+from workloads import gen
+
+pytestmark = pytest.mark.gpu
+
+F32, RESID, SWIGLU = 0, 1, 2
+
+
+@pytest.fixture(scope="module")
+def S():
+    assert torch.cuda.is_available(), "GPU test run without a GPU"
+    from paper_2609_36590_gb300 import build
+    build.build()
+    import paper_2609_36590_gb300 as s
+    return s
+
+
+def dev16(bits):
+    return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).cuda().view(torch.bfloat16)
+
+
+def host16(t):
+    return t.view(torch.int16).cpu().numpy().view(np.uint16)
+
+
+def bits(g, shape, s=1.0):
+    return gen.f32_to_bf16_bits((g.standard_normal(shape) * s).astype(np.float32))
+
+
+def f64(b):
+    return gen.bf16_bits_to_f64(b)
+
+
+def bf16_steps(got_bits, ref):
+    """Distance in bf16 steps between device bf16 values and the oracle's
+    (already bf16-valued) float64 values."""
+    ref_bits = gen.f32_to_bf16_bits(ref.astype(np.float32)).astype(np.int64)
+    g = got_bits.astype(np.int64)
+    # order-preserving integer view of bf16
+    key = lambda u: np.where(u & 0x8000, 0x8000 - (u & 0x7FFF), 0x8000 + (u & 0x7FFF))
+    return np.abs(key(g) - key(ref_bits))
+
+
+LIN_CASES = [
+    # B, N, K, epilogue
+    (1, 300, 128, F32),        # every tile split over two CTAs
+    (3, 1000, 640, RESID),     # one unit per CTA, ten CTAs per tile
+    (17, 2560, 2560, F32),
+    (40, 700, 1024, SWIGLU),
+    (128, 512, 9728, RESID),   # tiles split over ~38 CTAs each
+    (64, 9728, 256, SWIGLU),
+    (33, 129, 64, F32),        # whole tiles, a one-row last tile
+    (96, 128 * 200, 64, F32),  # more tiles than CTAs
+]
+
+
+@pytest.mark.parametrize("case", LIN_CASES, ids=lambda c: "B{}_N{}_K{}_e{}".format(*c))
+def test_linear_matches_oracle(S, case):
+    B, N, K, epi = case
+    g = np.random.default_rng(B * 1000 + N + K)
+    xb = bits(g, (B, K))
+    wb = bits(g, (N, K), K ** -0.5)
+    w2b = bits(g, (N, K), K ** -0.5) if epi == SWIGLU else None
+    x, W = f64(xb), f64(wb)
+    ref = x @ W.T
+    bound = 1e-5 * (np.abs(x) @ np.abs(W).T) + 1e-6
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    ws = S.new_linear_workspace(B, N, K, epi)
+    if epi == SWIGLU:
+        y = torch.empty(B, N, dtype=torch.bfloat16, device="cuda")
+        up = x @ f64(w2b).T
+        want = DS.silu(ref) * up
+        S.seed_linear(dev16(xb), dev16(wb), y, ws, err, S.LINEAR_SWIGLU, w2=dev16(w2b))
+        got = f64(host16(y))
+        tol = 2.0 ** -8 * np.abs(want) + 1e-4 * (np.abs(DS.silu(ref)) * np.abs(up)) + \
+            2e-5 * bound * (1 + np.abs(up))
+        assert (np.abs(got - want) <= tol + 1e-6).all()
+    else:
+        y0 = g.standard_normal((B, N)).astype(np.float32) if epi == RESID else np.zeros((B, N), np.float32)
+        y = torch.from_numpy(y0.copy()).cuda()
+        S.seed_linear(dev16(xb), dev16(wb), y, ws, err, epi)
+        got = y.cpu().numpy().astype(np.float64)
+        want = y0.astype(np.float64) + ref
+        diff = np.abs(got - want)
+        assert (diff <= bound + 1e-6 * np.abs(want)).all(), f"max excess {np.max(diff - bound):.3g}"
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0
+    cnt = ws[:4 * 4096].view(torch.int32).cpu().numpy()
+    assert (cnt == 0).all(), "counters not zero after the call"
+    # determinism: same inputs, same bits
+    if epi == F32:
+        y2 = torch.zeros_like(y)
+        S.seed_linear(dev16(xb), dev16(wb), y2, ws, err, epi)
+        assert torch.equal(y, y2)
+
+
+def test_linear_workspace_shared_across_sizes(S):
+    """One workspace serves calls of different sizes in sequence (a decoder
+    layer runs four products on one): each call leaves the counters zero."""
+    B = 4
+    shapes = [(6144, 256, F32), (9728, 256, SWIGLU), (256, 9728, RESID), (2560, 512, F32)]
+    ws = torch.zeros(max(S.new_linear_workspace(B, n, k, e).numel() for n, k, e in shapes),
+                     dtype=torch.uint8, device="cuda")
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    g = np.random.default_rng(21)
+    for n, k, e in shapes:
+        xb, wb, w2b = bits(g, (B, k)), bits(g, (n, k), k ** -0.5), bits(g, (n, k), k ** -0.5)
+        ref = f64(xb) @ f64(wb).T
+        if e == SWIGLU:
+            y = torch.empty(B, n, dtype=torch.bfloat16, device="cuda")
+            S.seed_linear(dev16(xb), dev16(wb), y, ws, err, e, w2=dev16(w2b))
+            want = DS.silu(ref) * (f64(xb) @ f64(w2b).T)
+            got = f64(host16(y))
+            assert (np.abs(got - want) <= 2.0 ** -7 * np.abs(want) + 1e-3).all()
+        else:
+            y = torch.zeros(B, n, device="cuda")
+            S.seed_linear(dev16(xb), dev16(wb), y, ws, err, e)
+            assert np.abs(y.cpu().numpy() - ref).max() <= 1e-4 * np.abs(ref).max()
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0
+
+
+def test_embed_and_rmsnorm(S):
+    g = np.random.default_rng(5)
+    V, d, B = 1000, 320, 6
+    wb = bits(g, (V, d))
+    tokens = np.array([0, 999, 17, 17, 500, 3], dtype=np.int32)
+    x = torch.empty(B, d, device="cuda")
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    S.seed_embed(torch.from_numpy(tokens).cuda(), dev16(wb), x, err)
+    np.testing.assert_array_equal(x.cpu().numpy().astype(np.float64), f64(wb)[tokens])
+    gamma = bits(g, (d,), 0.3)
+    xs = (g.standard_normal((B, d)) * 5).astype(np.float32)
+    y = torch.empty(B, d, dtype=torch.bfloat16, device="cuda")
+    S.seed_rmsnorm(torch.from_numpy(xs).cuda(), dev16(gamma), 1e-6, y)
+    ref = DS.bf16_round(DS.rms_norm(xs.astype(np.float64), f64(gamma)))
+    assert bf16_steps(host16(y), ref).max() <= 1
+    # an out-of-range token raises the device flag and leaves its row alone
+    x.fill_(7.0)
+    S.seed_embed(torch.tensor([1, 1000, -1, 2], dtype=torch.int32, device="cuda"), dev16(wb),
+                 x[:4], err)
+    torch.cuda.synchronize()
+    assert int(err.item()) & 256
+    assert (x[1:3].cpu().numpy() == 7.0).all()
+
+
+def paged_cache(rows, lens, pt, num_pages, hkv, D):
+    cache = np.full((num_pages, hkv, 16, D), gen.BF16_NAN, dtype=np.uint16)
+    for b in range(rows.shape[0]):
+        pos = np.arange(int(lens[b]))
+        cache[pt[b, pos // 16], :, pos % 16] = rows[b, pos]
+    return cache
+
+
+def make_layer_bits(g, dm, F_, hq, hkv, D):
+    one = lambda n, s: gen.f32_to_bf16_bits((1.0 + g.standard_normal(n) * s).astype(np.float32))
+    return dict(g_attn=one(dm, 0.2), w_qkv=bits(g, ((hq + 2 * hkv) * D, dm), dm ** -0.5),
+                g_q=one(D, 0.2), g_k=one(D, 0.2), w_o=bits(g, (dm, hq * D), (hq * D) ** -0.5),
+                g_mlp=one(dm, 0.2), w_gate=bits(g, (F_, dm), dm ** -0.5),
+                w_up=bits(g, (F_, dm), dm ** -0.5), w_down=bits(g, (dm, F_), F_ ** -0.5))
+
+
+def oracle_params(Lb):
+    return dict(g_attn=f64(Lb["g_attn"]), Wqkv=f64(Lb["w_qkv"]), g_q=f64(Lb["g_q"]),
+                g_k=f64(Lb["g_k"]), Wo=f64(Lb["w_o"]), g_mlp=f64(Lb["g_mlp"]),
+                Wg=f64(Lb["w_gate"]), Wu=f64(Lb["w_up"]), Wd=f64(Lb["w_down"]))
+
+
+class LayerCase:
+    """One decoder layer's cache, draft scratch and weights on both sides."""
+
+    def __init__(self, S, seed, B, dm, F_, hq, hkv, D, kmax, max_ctx, lens=None, dls=None):
+        g = np.random.default_rng(seed)
+        self.B, self.hq, self.hkv, self.D = B, hq, hkv, D
+        self.lens = (g.integers(0, max_ctx + 1, B) if lens is None else np.array(lens)).astype(np.int32)
+        self.dls = (g.integers(1, kmax + 1, B) if dls is None else np.array(dls)).astype(np.int32)
+        n_rows = max_ctx + 1
+        self.max_pages = -(-n_rows // 16) + 1
+        pt = g.permutation(B * self.max_pages).reshape(B, self.max_pages).astype(np.int32)
+        self.rows_k = bits(g, (B, n_rows, hkv, D))
+        self.rows_v = bits(g, (B, n_rows, hkv, D))
+        self.dk = bits(g, (B, hkv, kmax, D))
+        self.dv = bits(g, (B, hkv, kmax, D))
+        self.Lb = make_layer_bits(g, dm, F_, hq, hkv, D)
+        self.cfg = S.SeedConfig(hq=hq, hkv=hkv, head_dim=D, kmax=kmax)
+        num_pages = B * self.max_pages
+        self.kv = S.PagedKV(dev16(paged_cache(self.rows_k, self.lens, pt, num_pages, hkv, D)),
+                            dev16(paged_cache(self.rows_v, self.lens, pt, num_pages, hkv, D)),
+                            torch.from_numpy(pt).cuda())
+        self.layer = S.DecoderLayer(**{k: dev16(v) for k, v in self.Lb.items()})
+        self.dk_dev, self.dv_dev = dev16(self.dk), dev16(self.dv)
+        self.ws = S.new_draft_layer_workspace(self.cfg, self.layer, B)
+
+    def oracle(self, x):
+        ctx_k = [f64(self.rows_k[b, :self.lens[b]]) for b in range(self.B)]
+        ctx_v = [f64(self.rows_v[b, :self.lens[b]]) for b in range(self.B)]
+        dk = [f64(self.dk[b, :, :max(self.dls[b] - 1, 0)].transpose(1, 0, 2)) for b in range(self.B)]
+        dv = [f64(self.dv[b, :, :max(self.dls[b] - 1, 0)].transpose(1, 0, 2)) for b in range(self.B)]
+        pos = self.lens + self.dls - 1
+        return DS.decoder_layer(x, oracle_params(self.Lb), pos, ctx_k, ctx_v, dk, dv, self.hq,
+                                self.hkv, self.D)
+
+    def run(self, S, x_dev, err):
+        S.seed_draft_layer(self.cfg, self.layer, x_dev, self.kv, torch.from_numpy(self.lens).cuda(),
+                           self.dk_dev, self.dv_dev, torch.from_numpy(self.dls).cuda(), self.ws, err)
+
+
+def check_layer(case, x0, x_dev):
+    act = case.dls > 0
+    xr, kr, vr, _ = case.oracle(x0)
+    got_x = x_dev.cpu().numpy().astype(np.float64)
+    scale = np.abs(xr[act]).max()
+    dx = np.abs(got_x[act] - xr[act]).max()
+    assert dx <= 5e-3 * scale, f"x: max abs err {dx:.3g} (scale {scale:.3g})"
+    dk, dv = host16(case.dk_dev), host16(case.dv_dev)
+    for b in np.nonzero(act)[0]:
+        r = case.dls[b] - 1
+        for got, ref in ((dk[b, :, r], kr[b]), (dv[b, :, r], vr[b])):
+            st = bf16_steps(got, ref)
+            assert st.max() <= 1 and (st > 0).mean() <= 0.01, f"draft row b={b}: {st.max()}"
+        # rows other than r are untouched
+        others = [j for j in range(dk.shape[2]) if j != r]
+        np.testing.assert_array_equal(dk[b][:, others], case.dk[b][:, others])
+    return xr
+
+
+@pytest.mark.parametrize("D", [64, 128])
+def test_draft_layer_matches_oracle(S, D):
+    B, dm, F_, hq, hkv, kmax = 6, 256, 448, 8, 2, 5
+    case = LayerCase(S, 30 + D, B, dm, F_, hq, hkv, D, kmax, 200,
+                     lens=[0, 1, 17, 150, 200, 33], dls=[1, 3, 5, 0, 2, 4])
+    g = np.random.default_rng(7)
+    x0 = (g.standard_normal((B, dm)) * 2.0).astype(np.float32)
+    x_dev = torch.from_numpy(x0.copy()).cuda()
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    case.run(S, x_dev, err)
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0
+    check_layer(case, x0.astype(np.float64), x_dev)
+
+
+def test_draft_step_at_4b_scale(S):
+    """Qwen3-4B-sized drafter (d_model 2560, d_ff 9728, 32 q / 8 KV heads of
+    128, vocab 151936, tied embedding): embedding, two decoder layers, final
+    norm and the dynamic-drafting head for 4 sequences at draft step 2."""
+    B, dm, F_, hq, hkv, D, kmax, V = 4, 2560, 9728, 32, 8, 128, 4, 151936
+    g = np.random.default_rng(99)
+    lens, dls = [700, 64, 1029, 300], [2, 2, 2, 2]
+    cases = [LayerCase(S, 200 + l, B, dm, F_, hq, hkv, D, kmax, 1100, lens=lens, dls=dls)
+             for l in range(2)]
+    w_emb = bits(g, (V, dm), 0.02)
+    g_final = gen.f32_to_bf16_bits((1.0 + g.standard_normal(dm) * 0.2).astype(np.float32))
+    tokens = np.array([5, 151935, 77, 12345], dtype=np.int32)
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    x = torch.empty(B, dm, device="cuda")
+    W = dev16(w_emb)
+    S.seed_embed(torch.from_numpy(tokens).cuda(), W, x, err)
+    xr = f64(w_emb)[tokens]
+    for c in cases:
+        x_in = x.cpu().numpy().astype(np.float64)
+        c.run(S, x, err)
+        torch.cuda.synchronize()
+        check_layer(c, x_in, x)
+        # the device continues from its own x; the oracle's reference chain
+        # is carried separately so errors cannot compound silently
+        xr, _, _, _ = c.oracle(xr)
+        assert np.abs(x.cpu().numpy() - xr).max() <= 1e-2 * np.abs(xr).max()
+    h = torch.empty(B, dm, dtype=torch.bfloat16, device="cuda")
+    S.seed_rmsnorm(x, dev16(g_final), 1e-6, h)
+    href = DS.bf16_round(DS.rms_norm(xr, f64(g_final)))
+    assert np.abs(f64(host16(h)) - href).max() <= 1e-2 * np.abs(href).max()
+    ids = torch.empty(B, 10, dtype=torch.int32, device="cuda")
+    probs = torch.empty(B, 10, device="cuda")
+    ns = torch.empty(B, dtype=torch.int32, device="cuda")
+    stop = torch.empty(B, dtype=torch.int32, device="cuda")
+    lse = torch.empty(B, device="cuda")
+    S.seed_draft_head_topk(h, W, 0.7, ids, probs, ns, stop, lse,
+                           S.new_draft_head_workspace(B), err)
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0
+    # the head on the device's h against the oracle's head on the same h
+    o_ids, o_probs, _, _, _, o_lse = OD.draft_head(f64(host16(h)), f64(w_emb), 0.7)
+    np.testing.assert_allclose(lse.cpu().numpy(), o_lse, rtol=0, atol=2e-3)
+    np.testing.assert_allclose(probs.cpu().numpy()[:, 0], o_probs[:, 0], rtol=1e-2, atol=2e-3)
+    # and the head on the oracle's own h: same top token for these sequences
+    # wherever its probability is clear of the runner-up
+    r_ids, r_probs, _, _, _, _ = OD.draft_head(href, f64(w_emb), 0.7)
+    clear = r_probs[:, 0] - r_probs[:, 1] > 1e-2
+    np.testing.assert_array_equal(ids.cpu().numpy()[clear, 0], r_ids[clear, 0])
