@@ -376,6 +376,9 @@ def run_profile(args):
     if args.profile == "head":
         run_profile_head(args, wl, args.head_batch)
         return
+    if args.profile == "draftstep":
+        run_profile_draftstep(args, wl)
+        return
     dw = DeviceWorkload(wl, device="cuda:0", layers=list(wl.dec_layers), rounds=2)
     ins = dw.round_inputs(0)
     k_b = ins["k_b_np"]
@@ -473,6 +476,106 @@ def run_profile_head(args, wl, batch=None):
                       "alg_bytes_per_launch": nbytes, "us_median": round(med, 1),
                       "achieved_gbs": round(gbs, 1), "peak_gbs": peak, "peak_kind": kind,
                       "frac": round(gbs / peak, 3), "us": [round(u, 1) for u in us]}))
+
+
+DRAFTER = dict(d_model=2560, d_ff=9728)   # Qwen3-4B decoder layers
+
+
+def drafter_bytes(wl) -> int:
+    """Weight bytes one draft step reads: per decoder layer W_qkv, W_o,
+    W_gate, W_up, W_down and three norm gains, plus the tied head."""
+    dm, F, D = DRAFTER["d_model"], DRAFTER["d_ff"], wl.head_dim
+    per_layer = (wl.hq + 2 * wl.hkv) * D * dm + dm * wl.hq * D + 3 * F * dm + 2 * dm + 2 * D
+    return 2 * (len(wl.dec_layers) * per_layer + HEAD_VOCAB * dm + dm)
+
+
+def run_profile_draftstep(args, wl):
+    """--profile draftstep: one whole draft step of the workload's batch on the
+    device -- embedding, the two decoder layers (norms, QKV, q/k norm + RoPE,
+    draft KV append, draft attention over the layer's cache, output product,
+    SwiGLU MLP), final norm and the dynamic-drafting head -- with random
+    bf16 weights of a Qwen3-4B drafter, replayed `--reps` times from one CUDA
+    graph.  Algorithmic bytes: the drafter's weights once, plus each decoder
+    layer's draft attention bytes (its visible K/V rows, q, o).  Weights and
+    caches (GBs) are far above the L2 size."""
+    import torch
+
+    import paper_2609_36590_gb300 as seed
+    from workloads.device import DeviceWorkload
+
+    dev = "cuda:0"
+    dw = DeviceWorkload(wl, device=dev, layers=list(wl.dec_layers), rounds=2)
+    ins = dw.round_inputs(0)
+    B, dm, F, D = wl.batch, DRAFTER["d_model"], DRAFTER["d_ff"], wl.head_dim
+    g = torch.Generator(device=dev).manual_seed(20261)
+
+    def w(*shape, s=1.0):
+        return (torch.randn(*shape, device=dev, generator=g) * s).to(torch.bfloat16)
+
+    def gain(n):
+        return (1.0 + 0.1 * torch.randn(n, device=dev, generator=g)).to(torch.bfloat16)
+
+    layers = {l: seed.DecoderLayer(
+        g_attn=gain(dm), w_qkv=w((wl.hq + 2 * wl.hkv) * D, dm, s=dm ** -0.5), g_q=gain(D),
+        g_k=gain(D), w_o=w(dm, wl.hq * D, s=(wl.hq * D) ** -0.5), g_mlp=gain(dm),
+        w_gate=w(F, dm, s=dm ** -0.5), w_up=w(F, dm, s=dm ** -0.5), w_down=w(dm, F, s=F ** -0.5))
+        for l in wl.dec_layers}
+    w_emb = w(HEAD_VOCAB, dm, s=0.02)
+    g_final = gain(dm)
+    tokens = torch.randint(0, HEAD_VOCAB, (B,), device=dev, generator=g, dtype=torch.int32)
+    draft_lens = ins["draft_lens"][0]          # step 1 of round 0 (ragged k: some skip)
+    x = torch.empty(B, dm, device=dev)
+    h = torch.empty(B, dm, dtype=torch.bfloat16, device=dev)
+    ids = torch.empty(B, 10, dtype=torch.int32, device=dev)
+    probs = torch.empty(B, 10, device=dev)
+    n_sib = torch.empty(B, dtype=torch.int32, device=dev)
+    stop = torch.empty(B, dtype=torch.int32, device=dev)
+    lse = torch.empty(B, device=dev)
+    ws = seed.new_draft_layer_workspace(dw.cfg, layers[wl.dec_layers[0]], B, dev)
+    hws = seed.new_draft_head_workspace(B, dev)
+    err = dw.err
+
+    def step():
+        seed.seed_embed(tokens, w_emb, x, err)
+        for l in wl.dec_layers:
+            seed.seed_draft_layer(dw.cfg, layers[l], x, dw.kv[l], dw.ctx_lens, dw.draft_k[l],
+                                  dw.draft_v[l], draft_lens, ws, err)
+        seed.seed_rmsnorm(x, g_final, 1e-6, h)
+        seed.seed_draft_head_topk(h, w_emb, 0.7, ids, probs, n_sib, stop, lse, hws, err)
+
+    s = torch.cuda.Stream(device=dev)
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        for _ in range(3):
+            step()
+    torch.cuda.current_stream().wait_stream(s)
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        step()
+    for _ in range(3):
+        graph.replay()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.reps + 1)]
+    torch.cuda.synchronize()
+    ev[0].record()
+    for r in range(args.reps):
+        graph.replay()
+        ev[r + 1].record()
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0, "device error flag raised"
+    k_b = ins["k_b_np"]
+    attn = sum(attn_call_bytes(wl, "draft", (1, l), dw.lens0, k_b) for l in wl.dec_layers)
+    nbytes = drafter_bytes(wl) + attn
+    us = [ev[i].elapsed_time(ev[i + 1]) * 1e3 for i in range(args.reps)]
+    med = float(np.median(us))
+    peak, kind = load_peaks()
+    gbs = nbytes / med / 1e3
+    print(json.dumps({"profile": "draftstep", "workload": wl.name, "batch": B,
+                      "active": int((draft_lens > 0).sum().item()), "d_model": dm, "d_ff": F,
+                      "vocab": HEAD_VOCAB, "weight_bytes": drafter_bytes(wl),
+                      "attn_bytes": attn, "alg_bytes_per_step": nbytes,
+                      "us_median": round(med, 1), "achieved_gbs": round(gbs, 1),
+                      "peak_gbs": peak, "peak_kind": kind, "frac": round(gbs / peak, 3),
+                      "us": [round(u, 1) for u in us]}))
 
 
 def aggregate(rank_bytes: float, rank_seconds: float, world: int, device="cpu"):
@@ -592,7 +695,8 @@ def main():
     ap.add_argument("--impl", default="seed", choices=["seed", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=12.0)
-    ap.add_argument("--profile", choices=["draft", "verify", "tree", "head"], default=None,
+    ap.add_argument("--profile", choices=["draft", "verify", "tree", "head", "draftstep"],
+                    default=None,
                     help="launch one attention kind a few times for an ncu capture")
     ap.add_argument("--reps", type=int, default=3)
     ap.add_argument("--head-batch", type=int, default=None,

@@ -323,15 +323,18 @@ seed_status_t seed_draft_head_topk(int32_t batch, int32_t d_model, int32_t vocab
 #define SEED_LINEAR_SWIGLU    2  /* y  = bf16(silu(x W^T) * (x W2^T)), bf16 [batch, n_out] */
 #define SEED_LINEAR_MAX_BATCH 128
 
-/* Workspace bytes of seed_linear for these sizes and epilogue on the current
- * device: a fixed block of per-tile arrival counters, then stream-K partial
- * sums.  It must be 256-byte aligned and ZERO-FILLED before its first use;
- * every call leaves the counters zero again, so one workspace (of the largest
- * size needed) serves any sequence of calls on one stream.  0 for sizes
- * seed_linear rejects. */
+/* Workspace bytes of seed_linear for these sizes and epilogue: a fixed block
+ * of per-tile arrival counters, then an f32 scratch of (1, or 2 for SwiGLU)
+ * x batch x n_out sums.  It must be 256-byte aligned and ZERO-FILLED before
+ * its first use; every call leaves all of it zero again, so one workspace (of
+ * the largest size needed) serves any sequence of calls on one stream.  0 for
+ * sizes seed_linear rejects. */
 size_t seed_linear_workspace_bytes(int32_t batch, int32_t n_out, int32_t k_in, int32_t epilogue);
 
-/* y (epilogue) x W^T on the tensor cores, one pass over W.
+/* y (epilogue) x W^T on the tensor cores, one pass over W.  Work is split
+ * evenly over the SMs by (128-row tile, 64-wide K slab); a tile whose slabs
+ * fall on several CTAs is summed in f32 with atomic adds, so its last bits
+ * can differ between runs (tiles computed whole are bit-reproducible).
  *   x      bf16 [batch, k_in], batch in [1, SEED_LINEAR_MAX_BATCH], k_in % 64 == 0,
  *          n_out <= 524288
  *   w      bf16 [n_out, k_in]; w2 bf16 [n_out, k_in] for SEED_LINEAR_SWIGLU

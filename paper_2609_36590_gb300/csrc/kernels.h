@@ -126,7 +126,7 @@ constexpr size_t kLinearCntBytes = kLinearMaxTiles * sizeof(int32_t);
 enum LinearEpi : int32_t { kEpiF32 = 0, kEpiResidF32 = 1, kEpiSwigluBf16 = 2 };
 struct LinearParams {
   void* y;            // f32 [B, N] (kEpiF32, kEpiResidF32) or bf16 [B, N] (kEpiSwigluBf16)
-  float* part;        // [ctas * 2, (1|2) * nb, 128] partial accumulators
+  float* acc;         // [(1|2), B, N] f32 scratch for tiles split over CTAs, zero between calls
   int32_t* cnt;       // [kLinearMaxTiles] arrival counters, zero between calls
   int32_t* err;
   int32_t B, K, N, epi;

@@ -10,9 +10,10 @@
 // (tile, slab) units of the whole product are cut into equal contiguous
 // ranges, one per CTA, so every SM streams the same number of bytes whatever
 // N and K are.  A tile whose slabs span several CTAs is finished by the last
-// of them to arrive: each writes its partial accumulator to the workspace,
-// bumps the tile's counter, and the one that completes it sums the partials,
-// applies the epilogue and zeroes the counter again.
+// of them to arrive: each adds its share to an f32 scratch with atomic adds
+// (so the split sum's order, and its last bits, may vary between runs), bumps
+// the tile's counter, and the one that completes it applies the epilogue to
+// the sums and zeroes the scratch and the counter again.
 //
 // Epilogues: y = acc (f32); y += acc (f32 residual stream); and SwiGLU, where
 // a second weight matrix (the up projection) runs as a second MMA on the same
@@ -287,7 +288,7 @@ __global__ void __launch_bounds__(kLThreads, 1) linear_tc_kernel(
     const int q = warp;
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
     const int row = q * 32 + lane;
-    const int ncol = NW * nb;
+    const size_t accn = (size_t)p.B * p.N;   // one matrix's accumulator in the scratch
     bool ok = true;
     int t = t_first, k = k_first;
     for (int n = 0; t <= t_last; ++t, k = 0, ++n) {
@@ -298,8 +299,6 @@ __global__ void __launch_bounds__(kLThreads, 1) linear_tc_kernel(
       const uint32_t col0 = tmem + lane_off + (uint32_t)(n & 1) * bufcols;
       const int nrow = t * kLRows + row;
       const bool vrow = nrow < p.N;
-      const int slot = t == t_first ? 0 : 1;
-      float* pp = p.part + (size_t)(blockIdx.x * 2 + slot) * ncol * kLRows;
 #pragma unroll
       for (int c = 0; c < NCH; ++c) {
         uint32_t rg[32], ru[32];
@@ -312,24 +311,28 @@ __global__ void __launch_bounds__(kLThreads, 1) linear_tc_kernel(
             __syncwarp();
             if (lane == 0) mbar_arrive(&ctrl->d_empty[n & 1]);
           }
+          if (vrow) {
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const int b = c * 32 + i;
-            if (b < p.B) {
-              const float g = __uint_as_float(rg[i]);
-              const float u = NW == 2 ? __uint_as_float(ru[i]) : 0.f;
-              if (whole) {
-                if (vrow) finish_one<NW>(p, b, nrow, g, u);
-              } else {
-                pp[(size_t)b * kLRows + row] = g;
-                if (NW == 2) pp[(size_t)(nb + b) * kLRows + row] = u;
+            for (int i = 0; i < 32; ++i) {
+              const int b = c * 32 + i;
+              if (b < p.B) {
+                const float g = __uint_as_float(rg[i]);
+                const float u = NW == 2 ? __uint_as_float(ru[i]) : 0.f;
+                if (whole) {
+                  finish_one<NW>(p, b, nrow, g, u);
+                } else {
+                  // a share of a tile split over CTAs: add it to the scratch
+                  atomicAdd(p.acc + (size_t)b * p.N + nrow, g);
+                  if (NW == 2) atomicAdd(p.acc + accn + (size_t)b * p.N + nrow, u);
+                }
               }
             }
           }
         }
       }
       if (whole) continue;
-      // a tile shared with other CTAs: the last to arrive finishes it
+      // the last CTA of the tile to arrive applies the epilogue to the sums
+      // and leaves the scratch zeroed
       __threadfence();
       epi_bar();
       if (tid == 0) {
@@ -341,18 +344,24 @@ __global__ void __launch_bounds__(kLThreads, 1) linear_tc_kernel(
       epi_bar();
       if (ctrl->last) {
         __threadfence();
-        const int cf = lin_cta_of(U, (long long)t * nslab, nct);
-        const int cl = lin_cta_of(U, (long long)(t + 1) * nslab - 1, nct);
         if (vrow) {
-          for (int b = 0; b < p.B; ++b) {
-            float g = 0.f, u = 0.f;
-            for (int c = cf; c <= cl; ++c) {
-              const int sl = (lin_start(U, c, nct) / nslab) == t ? 0 : 1;
-              const float* src = p.part + (size_t)(c * 2 + sl) * ncol * kLRows;
-              g += src[(size_t)b * kLRows + row];
-              if (NW == 2) u += src[(size_t)(nb + b) * kLRows + row];
+          for (int b0 = 0; b0 < p.B; b0 += 32) {
+            float g[32], u[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const size_t at = (size_t)(b0 + i) * p.N + nrow;
+              g[i] = b0 + i < p.B ? __ldcg(p.acc + at) : 0.f;
+              u[i] = NW == 2 && b0 + i < p.B ? __ldcg(p.acc + accn + at) : 0.f;
             }
-            finish_one<NW>(p, b, nrow, g, u);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              if (b0 + i < p.B) {
+                const size_t at = (size_t)(b0 + i) * p.N + nrow;
+                finish_one<NW>(p, b0 + i, nrow, g[i], u[i]);
+                p.acc[at] = 0.f;
+                if (NW == 2) p.acc[accn + at] = 0.f;
+              }
+            }
           }
         }
         if (tid == 0) p.cnt[t] = 0;           // the workspace stays zeroed
@@ -431,11 +440,12 @@ int linear_ctas(int32_t n_out, int32_t k_in) {
 }
 
 // Workspace: a fixed prefix of kLinearMaxTiles counters (so that calls of any
-// size can share one workspace), then the partial accumulators.
+// size can share one workspace), then the f32 scratch [nw][batch][n_out].
+// Both are zero between calls.
 size_t linear_workspace_bytes(int32_t batch, int32_t n_out, int32_t k_in, int32_t epi) {
   const int nw = epi == kEpiSwigluBf16 ? 2 : 1;
-  return kLinearCntBytes +
-         (size_t)linear_ctas(n_out, k_in) * 2 * nw * lin_nb(batch) * kLRows * sizeof(float);
+  (void)k_in;
+  return kLinearCntBytes + (size_t)nw * batch * n_out * sizeof(float);
 }
 
 cudaError_t launch_linear(LinearParams prm, const void* x, const void* w, const void* w2, void* ws,
@@ -443,7 +453,7 @@ cudaError_t launch_linear(LinearParams prm, const void* x, const void* w, const 
   const int nw = prm.epi == kEpiSwigluBf16 ? 2 : 1;
   const int nb = lin_nb(prm.B);
   prm.cnt = static_cast<int32_t*>(ws);
-  prm.part = reinterpret_cast<float*>(static_cast<char*>(ws) + kLinearCntBytes);
+  prm.acc = reinterpret_cast<float*>(static_cast<char*>(ws) + kLinearCntBytes);
   CUtensorMap tx, tw, tw2;
   if (!encode_rows(&tx, x, (uint64_t)prm.K, (uint64_t)prm.B, (uint32_t)nb))
     return cudaErrorInvalidValue;

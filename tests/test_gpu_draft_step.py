@@ -5,7 +5,7 @@ model's last layers) through the C ABI against the oracle:
   split tiles across many CTAs (stream-K partials and last-arriver sums),
   ragged row tiles and every batch class: within the float32-accumulation
   bound of the exact float64 product (and half a bf16 step for SwiGLU);
-  deterministic, and the workspace counters are zero again afterwards;
+  whole tiles bit-reproducible, and the workspace zero again afterwards;
 * seed_embed (exact) and seed_rmsnorm (within one bf16 step);
 * seed_draft_layer for head_dim 64 and 128 against the oracle's layer
   (which rounds the same operands to bf16): the appended draft K/V rows and
@@ -115,10 +115,9 @@ def test_linear_matches_oracle(S, case):
         assert (diff <= bound + 1e-6 * np.abs(want)).all(), f"max excess {np.max(diff - bound):.3g}"
     torch.cuda.synchronize()
     assert int(err.item()) == 0
-    cnt = ws[:4 * 4096].view(torch.int32).cpu().numpy()
-    assert (cnt == 0).all(), "counters not zero after the call"
-    # determinism: same inputs, same bits
-    if epi == F32:
+    assert not ws.any().item(), "workspace not zero after the call"
+    # tiles computed whole (one K slab here) are bit-reproducible
+    if epi == F32 and K == 64:
         y2 = torch.zeros_like(y)
         S.seed_linear(dev16(xb), dev16(wb), y2, ws, err, epi)
         assert torch.equal(y, y2)
