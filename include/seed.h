@@ -348,13 +348,15 @@ seed_status_t seed_linear(int32_t batch, int32_t k_in, int32_t n_out, const void
                           void* ws, size_t ws_bytes, int32_t* err_flag, void* stream);
 
 /* x[b] = W_emb[tokens[b]] as f32 [batch, d_model] (the raw embedding H^0 the
- * drafter is fed, Sec. 4.1).  W_emb bf16 [vocab, d_model].
+ * drafter is fed, Sec. 4.1).  W_emb bf16 [vocab, d_model] (8-byte aligned),
+ * x 16-byte aligned, d_model % 4 == 0.
  * Device errors: SEED_DEVERR_TOKEN (that row is left untouched). */
 seed_status_t seed_embed(int32_t batch, int32_t d_model, int32_t vocab, const int32_t* tokens,
                          const void* w_emb, float* x, int32_t* err_flag, void* stream);
 
-/* y = bf16(x / sqrt(mean(x^2) + eps) * gamma) row by row; x f32 [rows, n],
- * gamma bf16 [n], y bf16 [rows, n]. */
+/* y = bf16(x / sqrt(mean(x^2) + eps) * gamma) row by row; x f32 [rows, n]
+ * (16-byte aligned), gamma bf16 [n] and y bf16 [rows, n] (8-byte aligned),
+ * n % 4 == 0. */
 seed_status_t seed_rmsnorm(int32_t rows, int32_t n, const float* x, const void* gamma,
                            float eps, void* y, void* stream);
 

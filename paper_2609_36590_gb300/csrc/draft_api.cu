@@ -14,6 +14,7 @@ namespace {
 
 seed_status_t fin(cudaError_t e) { return e == cudaSuccess ? SEED_OK : SEED_ERR_CUDA; }
 bool mis16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) != 0; }
+bool mis8(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 7u) != 0; }
 size_t up256(size_t n) { return (n + 255) & ~(size_t)255; }
 
 bool linear_shape_ok(int32_t batch, int32_t n_out, int32_t k_in, int32_t epi) {
@@ -97,18 +98,20 @@ seed_status_t seed_linear(int32_t batch, int32_t k_in, int32_t n_out, const void
 
 seed_status_t seed_embed(int32_t batch, int32_t d_model, int32_t vocab, const int32_t* tokens,
                          const void* w_emb, float* x, int32_t* err_flag, void* stream) {
-  if (batch < 0 || d_model <= 0 || vocab <= 0) return SEED_ERR_SHAPE;
+  if (batch < 0 || d_model <= 0 || d_model % 4 != 0 || vocab <= 0) return SEED_ERR_SHAPE;
   if (batch == 0) return SEED_OK;
   if (!tokens || !w_emb || !x || !err_flag) return SEED_ERR_NULL;
+  if (mis8(w_emb) || mis16(x)) return SEED_ERR_RANGE;
   return fin(seedk::launch_embed(batch, d_model, vocab, tokens, w_emb, x, err_flag,
                                  static_cast<cudaStream_t>(stream)));
 }
 
 seed_status_t seed_rmsnorm(int32_t rows, int32_t n, const float* x, const void* gamma, float eps,
                            void* y, void* stream) {
-  if (rows < 0 || n <= 0 || !(eps > 0.f)) return SEED_ERR_SHAPE;
+  if (rows < 0 || n <= 0 || n % 4 != 0 || !(eps > 0.f)) return SEED_ERR_SHAPE;
   if (rows == 0) return SEED_OK;
   if (!x || !gamma || !y) return SEED_ERR_NULL;
+  if (mis16(x) || mis8(gamma) || mis8(y)) return SEED_ERR_RANGE;
   return fin(seedk::launch_rmsnorm(rows, n, x, gamma, eps, y, static_cast<cudaStream_t>(stream)));
 }
 
@@ -134,7 +137,7 @@ seed_status_t seed_draft_layer(const seed_cfg_t* cfg, int32_t batch,
       !L.w_qkv || !L.g_q || !L.g_k || !L.w_o || !L.g_mlp || !L.w_gate || !L.w_up || !L.w_down)
     return SEED_ERR_NULL;
   if (mis16(L.w_qkv) || mis16(L.w_o) || mis16(L.w_gate) || mis16(L.w_up) || mis16(L.w_down) ||
-      mis16(x))
+      mis16(x) || mis8(L.g_attn) || mis8(L.g_mlp))
     return SEED_ERR_RANGE;
   const LayerWs w = layer_ws(cfg, layer, batch);
   if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0 || ws_bytes < w.total) return SEED_ERR_WORKSPACE;

@@ -8,6 +8,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <cmath>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -30,7 +31,8 @@ __device__ __forceinline__ float block_sum(float v, float* sh) {
   return t;
 }
 
-// x[b] = W_emb[tokens[b]] (bf16 -> f32).  One block per sequence.
+// x[b] = W_emb[tokens[b]] (bf16 -> f32).  One block per sequence; 8-byte
+// loads (d is a multiple of 4).
 __global__ void __launch_bounds__(kOpsThreads) embed_kernel(int32_t d, int32_t vocab,
                                                             const int32_t* tokens,
                                                             const __nv_bfloat16* w, float* x,
@@ -43,75 +45,125 @@ __global__ void __launch_bounds__(kOpsThreads) embed_kernel(int32_t d, int32_t v
     if (threadIdx.x == 0) raise_err(err, SEED_DEVERR_TOKEN);
     return;
   }
-  const __nv_bfloat16* row = w + (size_t)tok * d;
-  for (int i = threadIdx.x; i < d; i += blockDim.x)
-    x[(size_t)b * d + i] = __bfloat162float(row[i]);
+  const uint2* row = reinterpret_cast<const uint2*>(w + (size_t)tok * d);
+  float4* out = reinterpret_cast<float4*>(x + (size_t)b * d);
+  for (int i = threadIdx.x; i < d / 4; i += blockDim.x) {
+    const uint2 v = row[i];
+    out[i] = make_float4(__uint_as_float(v.x << 16), __uint_as_float(v.x & 0xffff0000u),
+                         __uint_as_float(v.y << 16), __uint_as_float(v.y & 0xffff0000u));
+  }
 }
 
-// y[b] = bf16(x[b] / sqrt(mean(x[b]^2) + eps) * gamma).  One block per row.
+// y[b] = bf16(x[b] / sqrt(mean(x[b]^2) + eps) * gamma).  One block per row;
+// a row of up to 4 * 4 * 256 floats stays in registers between the two
+// passes (longer rows read x twice).  n is a multiple of 4.
+constexpr int kNormVec = 4;                   // float4 per thread kept in registers
 __global__ void __launch_bounds__(kOpsThreads) rmsnorm_kernel(int32_t n, const float* x,
                                                               const __nv_bfloat16* gamma,
                                                               float eps, __nv_bfloat16* y) {
   __shared__ float sh[kOpsThreads / 32];
   if (threadIdx.x == 0) pdl_trigger();
   pdl_wait();
-  const float* xr = x + (size_t)blockIdx.x * n;
+  const float4* xr = reinterpret_cast<const float4*>(x + (size_t)blockIdx.x * n);
+  const int n4 = n / 4;
+  float4 v[kNormVec];
   float ss = 0.f;
-  for (int i = threadIdx.x; i < n; i += blockDim.x) ss = fmaf(xr[i], xr[i], ss);
+#pragma unroll
+  for (int j = 0; j < kNormVec; ++j) {
+    const int i = threadIdx.x + j * kOpsThreads;
+    v[j] = i < n4 ? xr[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+#pragma unroll
+  for (int j = 0; j < kNormVec; ++j)
+    ss += v[j].x * v[j].x + v[j].y * v[j].y + v[j].z * v[j].z + v[j].w * v[j].w;
+  for (int i = threadIdx.x + kNormVec * kOpsThreads; i < n4; i += kOpsThreads) {
+    const float4 u = xr[i];
+    ss += u.x * u.x + u.y * u.y + u.z * u.z + u.w * u.w;
+  }
   const float r = rsqrtf(block_sum(ss, sh) / (float)n + eps);
-  __nv_bfloat16* yr = y + (size_t)blockIdx.x * n;
-  for (int i = threadIdx.x; i < n; i += blockDim.x)
-    yr[i] = __float2bfloat16_rn(xr[i] * r * __bfloat162float(gamma[i]));
+  const uint2* gr = reinterpret_cast<const uint2*>(gamma);
+  uint2* yr = reinterpret_cast<uint2*>(y + (size_t)blockIdx.x * n);
+  auto put = [&](int i, float4 u) {
+    const uint2 g = gr[i];
+    const float2 lo = make_float2(u.x * r * __uint_as_float(g.x << 16),
+                                  u.y * r * __uint_as_float(g.x & 0xffff0000u));
+    const float2 hi = make_float2(u.z * r * __uint_as_float(g.y << 16),
+                                  u.w * r * __uint_as_float(g.y & 0xffff0000u));
+    const __nv_bfloat162 a = __float22bfloat162_rn(lo), c = __float22bfloat162_rn(hi);
+    yr[i] = make_uint2(*reinterpret_cast<const uint32_t*>(&a), *reinterpret_cast<const uint32_t*>(&c));
+  };
+#pragma unroll
+  for (int j = 0; j < kNormVec; ++j) {
+    const int i = threadIdx.x + j * kOpsThreads;
+    if (i < n4) put(i, v[j]);
+  }
+  for (int i = threadIdx.x + kNormVec * kOpsThreads; i < n4; i += kOpsThreads) put(i, xr[i]);
 }
 
 // From qkv f32 [B, (hq + 2 hkv) D]: q, k normed per head (gain g_q / g_k) and
 // rotated (rotate-half pairs (i, i + D/2), angle pos * theta^(-2i/D)); v
 // copied; all three rounded to bf16.  pos = ctx_len + draft_len - 1: the
-// position of the token this draft step feeds.  One block per sequence; the
-// angles are reduced in double precision (positions reach 10^5 and more).
-__global__ void __launch_bounds__(kOpsThreads) qk_norm_rope_kernel(
+// position of the token this draft step feeds.  One warp per (sequence,
+// head).  The frequencies theta^(-2i/D) come from the host in double; each
+// lane forms its angle pos * w in double and reduces it by 2 pi (split in two
+// doubles) before a single-precision sincos, so positions of 10^6 and more
+// keep their angles to ~1e-10 rad.
+constexpr int kRopeWarps = 8;
+struct RopeFreq {
+  double w[64];
+};
+__global__ void __launch_bounds__(kRopeWarps * 32) qk_norm_rope_kernel(
     int32_t hq, int32_t hkv, int32_t D, const float* qkv, const __nv_bfloat16* gq,
-    const __nv_bfloat16* gk, const int32_t* ctx_lens, const int32_t* draft_lens, float theta,
-    float eps, __nv_bfloat16* q, __nv_bfloat16* k, __nv_bfloat16* v) {
-  __shared__ float cs[64], sn[64];
+    const __nv_bfloat16* gk, const int32_t* ctx_lens, const int32_t* draft_lens,
+    const RopeFreq fr, float eps, __nv_bfloat16* q, __nv_bfloat16* k, __nv_bfloat16* v) {
   if (threadIdx.x == 0) pdl_trigger();
   pdl_wait();
   const int b = blockIdx.x;
-  const int dl = draft_lens[b];
-  if (dl <= 0) return;                        // skipped sequence
-  const long long pos = (long long)ctx_lens[b] + dl - 1;
-  const int half = D / 2;
-  for (int i = threadIdx.x; i < half; i += blockDim.x) {
-    const double inv = exp(-(2.0 * i / D) * log((double)theta));
-    double s, c;
-    sincos((double)pos * inv, &s, &c);
-    cs[i] = (float)c;
-    sn[i] = (float)s;
-  }
-  __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nh = hq + 2 * hkv;
-  const float* src = qkv + (size_t)b * nh * D;
-  for (int h = warp; h < nh; h += blockDim.x >> 5) {
-    const float* xh = src + (size_t)h * D;
-    if (h >= hq + hkv) {                      // v: copy
-      __nv_bfloat16* dst = v + ((size_t)b * hkv + (h - hq - hkv)) * D;
-      for (int i = lane; i < D; i += 32) dst[i] = __float2bfloat16_rn(xh[i]);
-      continue;
-    }
-    const bool isq = h < hq;
-    const __nv_bfloat16* g = isq ? gq : gk;
-    __nv_bfloat16* dst = isq ? q + ((size_t)b * hq + h) * D : k + ((size_t)b * hkv + (h - hq)) * D;
-    float ss = 0.f;
-    for (int i = lane; i < D; i += 32) ss = fmaf(xh[i], xh[i], ss);
+  const int h = blockIdx.y * kRopeWarps + warp;
+  if (h >= nh) return;
+  const int dl = draft_lens[b];
+  if (dl <= 0) return;                        // skipped sequence
+  const float* xh = qkv + ((size_t)b * nh + h) * D;
+  const int half = D / 2;                     // 32 or 64: one or two pairs per lane
+  if (h >= hq + hkv) {                        // v: copy
+    __nv_bfloat16* dst = v + ((size_t)b * hkv + (h - hq - hkv)) * D;
+    for (int i = lane; i < D; i += 32) dst[i] = __float2bfloat16_rn(xh[i]);
+    return;
+  }
+  const bool isq = h < hq;
+  const __nv_bfloat16* g = isq ? gq : gk;
+  __nv_bfloat16* dst = isq ? q + ((size_t)b * hq + h) * D : k + ((size_t)b * hkv + (h - hq)) * D;
+  const int np = half / 32;                   // pairs per lane
+  float a[2], c[2];
+  float ss = 0.f;
 #pragma unroll
-    for (int o = 16; o; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
-    const float r = rsqrtf(ss / (float)D + eps);
-    for (int i = lane; i < half; i += 32) {
-      const float a = xh[i] * r * __bfloat162float(g[i]);
-      const float c = xh[i + half] * r * __bfloat162float(g[i + half]);
-      dst[i] = __float2bfloat16_rn(a * cs[i] - c * sn[i]);
-      dst[i + half] = __float2bfloat16_rn(c * cs[i] + a * sn[i]);
+  for (int j = 0; j < 2; ++j) {
+    if (j < np) {
+      a[j] = xh[lane + 32 * j];
+      c[j] = xh[lane + 32 * j + half];
+      ss = fmaf(a[j], a[j], fmaf(c[j], c[j], ss));
+    }
+  }
+#pragma unroll
+  for (int o = 16; o; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  const float r = rsqrtf(ss / (float)D + eps);
+  const double pos = (double)((long long)ctx_lens[b] + dl - 1);
+  constexpr double kTwoPiHi = 6.283185307179586, kTwoPiLo = 2.4492935982947064e-16;
+#pragma unroll
+  for (int j = 0; j < 2; ++j) {
+    if (j < np) {
+      const int i = lane + 32 * j;
+      const double ang = pos * fr.w[i];
+      const double m = rint(ang * (1.0 / kTwoPiHi));
+      const float red = (float)fma(-m, kTwoPiLo, fma(-m, kTwoPiHi, ang));
+      float sn, cs;
+      sincosf(red, &sn, &cs);
+      const float x0 = a[j] * r * __bfloat162float(g[i]);
+      const float x1 = c[j] * r * __bfloat162float(g[i + half]);
+      dst[i] = __float2bfloat16_rn(x0 * cs - x1 * sn);
+      dst[i + half] = __float2bfloat16_rn(x1 * cs + x0 * sn);
     }
   }
 }
@@ -144,9 +196,12 @@ cudaError_t launch_qk_norm_rope(int32_t B, int32_t hq, int32_t hkv, int32_t D, c
                                 const void* gq, const void* gk, const int32_t* ctx_lens,
                                 const int32_t* draft_lens, float theta, float eps, void* q,
                                 void* k, void* v, cudaStream_t st) {
-  return launch_pdl(qk_norm_rope_kernel, dim3(B), dim3(kOpsThreads), 0, st, hq, hkv, D, qkv,
+  RopeFreq fr{};
+  for (int i = 0; i < D / 2 && i < 64; ++i) fr.w[i] = std::pow((double)theta, -2.0 * i / D);
+  const dim3 grid(B, (hq + 2 * hkv + kRopeWarps - 1) / kRopeWarps);
+  return launch_pdl(qk_norm_rope_kernel, grid, dim3(kRopeWarps * 32), 0, st, hq, hkv, D, qkv,
                     static_cast<const __nv_bfloat16*>(gq), static_cast<const __nv_bfloat16*>(gk),
-                    ctx_lens, draft_lens, theta, eps, static_cast<__nv_bfloat16*>(q),
+                    ctx_lens, draft_lens, fr, eps, static_cast<__nv_bfloat16*>(q),
                     static_cast<__nv_bfloat16*>(k), static_cast<__nv_bfloat16*>(v));
 }
 
