@@ -129,17 +129,30 @@ __device__ __forceinline__ void ldrain(uint64_t* bar, uint32_t parity, int32_t* 
 
 __device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 
-// The epilogue of one output element (b, n) from the finished accumulators.
+// The epilogue of 32 output elements (b0 + i, n), i < 32, b0 + i < B, from
+// the finished sums g (and u for SwiGLU).  For the residual epilogue all 32
+// old values are loaded before any store, so that their latencies overlap.
 template <int NW>
-__device__ __forceinline__ void finish_one(const LinearParams& p, int b, int n, float g, float u) {
-  const size_t i = (size_t)b * p.N + n;
+__device__ __forceinline__ void finish32(const LinearParams& p, int b0, int n, const float (&g)[32],
+                                         const float (&u)[32]) {
   if (NW == 2) {
-    const float s = g / (1.f + __expf(-g));
-    static_cast<__nv_bfloat16*>(p.y)[i] = __float2bfloat16_rn(s * u);
-  } else if (p.epi == kEpiResidF32) {
-    static_cast<float*>(p.y)[i] += g;
+    __nv_bfloat16* y = static_cast<__nv_bfloat16*>(p.y);
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      if (b0 + i < p.B) {
+        const float s = g[i] / (1.f + __expf(-g[i]));
+        y[(size_t)(b0 + i) * p.N + n] = __float2bfloat16_rn(s * u[i]);
+      }
+    }
   } else {
-    static_cast<float*>(p.y)[i] = g;
+    float* y = static_cast<float*>(p.y);
+    float old[32];
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+      old[i] = (p.epi == kEpiResidF32 && b0 + i < p.B) ? y[(size_t)(b0 + i) * p.N + n] : 0.f;
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+      if (b0 + i < p.B) y[(size_t)(b0 + i) * p.N + n] = old[i] + g[i];
   }
 }
 
@@ -312,18 +325,22 @@ __global__ void __launch_bounds__(kLThreads, 1) linear_tc_kernel(
             if (lane == 0) mbar_arrive(&ctrl->d_empty[n & 1]);
           }
           if (vrow) {
+            if (whole) {
+              float g[32], u[32];
 #pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const int b = c * 32 + i;
-              if (b < p.B) {
-                const float g = __uint_as_float(rg[i]);
-                const float u = NW == 2 ? __uint_as_float(ru[i]) : 0.f;
-                if (whole) {
-                  finish_one<NW>(p, b, nrow, g, u);
-                } else {
-                  // a share of a tile split over CTAs: add it to the scratch
-                  atomicAdd(p.acc + (size_t)b * p.N + nrow, g);
-                  if (NW == 2) atomicAdd(p.acc + accn + (size_t)b * p.N + nrow, u);
+              for (int i = 0; i < 32; ++i) {
+                g[i] = __uint_as_float(rg[i]);
+                u[i] = NW == 2 ? __uint_as_float(ru[i]) : 0.f;
+              }
+              finish32<NW>(p, c * 32, nrow, g, u);
+            } else {
+              // a share of a tile split over CTAs: add it to the scratch
+#pragma unroll
+              for (int i = 0; i < 32; ++i) {
+                const int b = c * 32 + i;
+                if (b < p.B) {
+                  atomicAdd(p.acc + (size_t)b * p.N + nrow, __uint_as_float(rg[i]));
+                  if (NW == 2) atomicAdd(p.acc + accn + (size_t)b * p.N + nrow, __uint_as_float(ru[i]));
                 }
               }
             }
@@ -353,11 +370,11 @@ __global__ void __launch_bounds__(kLThreads, 1) linear_tc_kernel(
               g[i] = b0 + i < p.B ? __ldcg(p.acc + at) : 0.f;
               u[i] = NW == 2 && b0 + i < p.B ? __ldcg(p.acc + accn + at) : 0.f;
             }
+            finish32<NW>(p, b0, nrow, g, u);
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
               if (b0 + i < p.B) {
                 const size_t at = (size_t)(b0 + i) * p.N + nrow;
-                finish_one<NW>(p, b0 + i, nrow, g[i], u[i]);
                 p.acc[at] = 0.f;
                 if (NW == 2) p.acc[accn + at] = 0.f;
               }
