@@ -24,6 +24,9 @@ the paper (SEED: Self-Speculative Decoding via Implicit Encoder-Decoder):
   the pre-norm form of the paper's Qwen3 models (RMS norms, q/k norms, RoPE,
   grouped attention over the deep cache plus the draft rows, SwiGLU MLP),
   final norm and the dynamic-drafting head.
+* ``block_attn`` -- the decoder's block-causal training attention (Sec. 3,
+  "Training with Block Attention"; Fig. 2): deep-cache rows of the preceding
+  blocks plus causal self-attention within the query's own block.
 * ``toy_model``  -- a tiny float64 transformer running Alg. 2 end to end (with
   a linear draft or a draft tree) and plain greedy decoding, for the
   exactness property of Sec. 4.1.
