@@ -402,6 +402,35 @@ seed_status_t seed_draft_layer(const seed_cfg_t* cfg, int32_t batch,
                                int32_t* err_flag, void* stream);
 
 /* ------------------------------------------------------------------------
+ * The decoder's block-causal training attention (Sec. 3, "Training with
+ * Block Attention"; Fig. 2, right), forward pass.  Sequences of n tokens are
+ * cut into blocks of b; the query at position p sees
+ *   - the deep keys/values k_dec/v_dec (the decoder layer's KV^dec from the
+ *     full forward pass) at every position < s(p) = (p / b) * b, and
+ *   - the layer's own keys/values over the raw embeddings, k_spec/v_spec,
+ *     at positions s(p) .. p (causal within the block).
+ *   cfg        hq, hkv, head_dim (64 or 128) and scale as for the other
+ *              calls; page_size and kmax are not used
+ *   n, block   n % block == 0, 2 <= block <= SEED_MAX_KMAX + 1 (a block of one
+ *              token is the draft call's shape: use seed_draft_attn)
+ *   q          bf16 [batch, n, hq, head_dim]
+ *   k_dec, v_dec, k_spec, v_spec   bf16 [batch, n, hkv, head_dim]
+ *   out        f32 [batch, n, hq, head_dim]; lse f32 [batch, n, hq] or NULL
+ *   ws         seed_block_attn_workspace_bytes(...) bytes, 256-byte aligned,
+ *              ZERO-FILLED before its first use (it holds the attention's
+ *              counters, which every call leaves zeroed, and a paged copy of
+ *              the rows that each call rewrites)
+ * Errors: SEED_ERR_SHAPE (sizes, block, head_dim, group), SEED_ERR_NULL,
+ * SEED_ERR_RANGE (a tensor not 16-byte aligned), SEED_ERR_WORKSPACE.
+ * Device errors: none expected (as seed_verify_attn). */
+size_t seed_block_attn_workspace_bytes(const seed_cfg_t* cfg, int32_t batch, int32_t n,
+                                       int32_t block);
+seed_status_t seed_block_attn(const seed_cfg_t* cfg, int32_t batch, int32_t n, int32_t block,
+                              const void* q, const void* k_dec, const void* v_dec,
+                              const void* k_spec, const void* v_spec, float* out, float* lse,
+                              void* ws, size_t ws_bytes, int32_t* err_flag, void* stream);
+
+/* ------------------------------------------------------------------------
  * Library convenience with no counterpart in the paper: verify attention
  * without a caller-provided workspace.
  *

@@ -12,7 +12,8 @@ seed_verify_attn_noalloc (verify attention on the library's built-in scratch,
 for callers that cannot provide a workspace), and the tree-verification calls
 seed_tree_verify_attn, seed_tree_accept_commit, seed_tree_kv_compact, the
 dynamic-drafting head seed_draft_head_topk, and the draft step on the device:
-seed_linear, seed_embed, seed_rmsnorm and seed_draft_layer.
+seed_linear, seed_embed, seed_rmsnorm and seed_draft_layer, and the decoder's
+block-causal training attention seed_block_attn.
 """
 
 from __future__ import annotations
@@ -80,6 +81,9 @@ _SIGS = {
                                                            ctypes.POINTER(_Layer), _I]),
     "seed_draft_layer": (_I, [ctypes.POINTER(_Cfg), _I, ctypes.POINTER(_Layer), _P, _KV, _P, _P,
                               _P, _P, _P, ctypes.c_size_t, _P, _P]),
+    "seed_block_attn_workspace_bytes": (ctypes.c_size_t, [ctypes.POINTER(_Cfg), _I, _I, _I]),
+    "seed_block_attn": (_I, [ctypes.POINTER(_Cfg), _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, _P,
+                             ctypes.c_size_t, _P, _P]),
     "seed_draft_head_topk": (_I, [_I, _I, _I, _P, _P, ctypes.c_float, _P, _P, _P, _P, _P, _P,
                                   ctypes.c_size_t, _P, _P]),
 }
@@ -452,6 +456,33 @@ def seed_draft_layer(cfg: SeedConfig, layer: DecoderLayer, x, ctx_kv: PagedKV, c
         _t(draft_v, torch.bfloat16, (B, cfg.hkv, cfg.kmax, cfg.head_dim), "draft_v"),
         _t(draft_lens, torch.int32, (B,), "draft_lens"), _t(ws, torch.uint8, None, "ws"),
         ws.numel(), _t(err, torch.int32, (1,), "err"), _stream(stream)))
+
+
+def new_block_attn_workspace(cfg: SeedConfig, batch: int, n: int, block: int,
+                             device=None) -> torch.Tensor:
+    c = cfg.c()
+    nb = _lib.seed_block_attn_workspace_bytes(ctypes.byref(c), batch, n, block)
+    if nb == 0:
+        raise SeedError("invalid seed_block_attn sizes")
+    return torch.zeros(int(nb), dtype=torch.uint8, device=device or "cuda")
+
+
+def seed_block_attn(cfg: SeedConfig, block: int, q, k_dec, v_dec, k_spec, v_spec, out, lse, ws,
+                    err, stream=None) -> None:
+    """Block-causal training attention: q bf16 [B, n, hq, D]; k/v_dec and
+    k/v_spec bf16 [B, n, hkv, D]; out f32 [B, n, hq, D]; lse f32 [B, n, hq]
+    or None."""
+    B, n = q.shape[0], q.shape[1]
+    kshape = (B, n, cfg.hkv, cfg.head_dim)
+    c = cfg.c()
+    _check(_lib.seed_block_attn(
+        ctypes.byref(c), B, n, block, _t(q, torch.bfloat16, (B, n, cfg.hq, cfg.head_dim), "q"),
+        _t(k_dec, torch.bfloat16, kshape, "k_dec"), _t(v_dec, torch.bfloat16, kshape, "v_dec"),
+        _t(k_spec, torch.bfloat16, kshape, "k_spec"), _t(v_spec, torch.bfloat16, kshape, "v_spec"),
+        _t(out, torch.float32, (B, n, cfg.hq, cfg.head_dim), "out"),
+        _t(lse, torch.float32, (B, n, cfg.hq), "lse") if lse is not None else None,
+        _t(ws, torch.uint8, None, "ws"), ws.numel(), _t(err, torch.int32, (1,), "err"),
+        _stream(stream)))
 
 
 def library() -> ctypes.CDLL:

@@ -219,3 +219,21 @@ def test_draft_layer_host_checks(lib):
     n = lib.seed_draft_layer_workspace_bytes(ctypes.byref(c), ctypes.byref(layer()), 4)
     assert n > lib.seed_workspace_bytes(ctypes.byref(c), 4)
     assert lib.seed_draft_layer_workspace_bytes(ctypes.byref(c), ctypes.byref(layer()), 0) == 0
+
+
+def test_block_attn_host_checks(lib):
+    c = _Cfg(32, 8, 128, 16, 8, 0.0)
+
+    def call(cf=c, B=2, n=40, b=10, q=FAKE, ws=FAKE, nbytes=1 << 34):
+        return lib.seed_block_attn(ctypes.byref(cf), B, n, b, q, FAKE, FAKE, FAKE, FAKE, FAKE,
+                                   None, ws, nbytes, FAKE, None)
+    assert call(B=0) == OK
+    assert call(n=41) == ERR_SHAPE               # n not a multiple of the block
+    assert call(b=33, n=66) == ERR_SHAPE         # block above kmax + 1 = 32
+    assert call(b=1, n=40) == ERR_SHAPE          # one-token blocks: the draft call's shape
+    assert call(cf=_Cfg(32, 8, 96, 16, 8, 0.0)) == ERR_SHAPE
+    assert call(q=None) == ERR_NULL
+    assert call(q=FAKE + 8) == ERR_RANGE
+    assert call(nbytes=4096) == ERR_WS
+    assert lib.seed_block_attn_workspace_bytes(ctypes.byref(c), 2, 40, 10) > 0
+    assert lib.seed_block_attn_workspace_bytes(ctypes.byref(c), 2, 41, 10) == 0
