@@ -379,6 +379,9 @@ def run_profile(args):
     if args.profile == "draftstep":
         run_profile_draftstep(args, wl)
         return
+    if args.profile == "blockattn":
+        run_profile_blockattn(args, wl)
+        return
     dw = DeviceWorkload(wl, device="cuda:0", layers=list(wl.dec_layers), rounds=2)
     ins = dw.round_inputs(0)
     k_b = ins["k_b_np"]
@@ -578,6 +581,59 @@ def run_profile_draftstep(args, wl):
                       "us": [round(u, 1) for u in us]}))
 
 
+def run_profile_blockattn(args, wl, n=1000, block=10, batch=8):
+    """--profile blockattn: the decoder's block-causal training attention
+    (Sec. 3) for `batch` sequences of n tokens in blocks of 10 (the paper's
+    training block size) at the workload's head shape, `--reps` calls back to
+    back.  Reports the bytes the implementation moves (each block's deep
+    prefix and own rows, q in, o and lse out, plus the paged copy it builds)
+    against the HBM peak, and the attention FLOPs."""
+    import torch
+
+    import paper_2609_36590_gb300 as seed
+
+    dev = "cuda:0"
+    hq, hkv, D = wl.hq, wl.hkv, wl.head_dim
+    g = torch.Generator(device=dev).manual_seed(20262)
+    q = torch.randn(batch, n, hq, D, device=dev, generator=g).to(torch.bfloat16)
+    kv = [torch.randn(batch, n, hkv, D, device=dev, generator=g).to(torch.bfloat16)
+          for _ in range(4)]
+    out = torch.empty(batch, n, hq, D, device=dev)
+    lse = torch.empty(batch, n, hq, device=dev)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    cfg = seed.SeedConfig(hq=hq, hkv=hkv, head_dim=D, kmax=1)
+    ws = seed.new_block_attn_workspace(cfg, batch, n, block, dev)
+    for _ in range(3):
+        seed.seed_block_attn(cfg, block, q, *kv, out, lse, ws, err)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(args.reps + 1)]
+    torch.cuda.synchronize()
+    ev[0].record()
+    for r in range(args.reps):
+        seed.seed_block_attn(cfg, block, q, *kv, out, lse, ws, err)
+        ev[r + 1].record()
+    torch.cuda.synchronize()
+    assert int(err.item()) == 0, "device error flag raised"
+    R = 2 * hkv * D * 2                               # K + V bytes of one row
+    nblk = n // block
+    rows_read = sum(s * block + block for s in range(nblk))      # deep prefix + own rows
+    pages = -(-n // 16) + nblk * -(-(15 + block) // 16)
+    copy = (n * 2 * R) + pages * 16 * R               # read 4 inputs, write the paged copy
+    qo = n * hq * (D * (2 + 4) + 4)
+    nbytes = batch * (rows_read * R + pages * 16 * R + copy + qo)
+    vis = sum(s * block + (j + 1) for s in range(nblk) for j in range(block))
+    flops = batch * hq * vis * D * 4
+    us = [ev[i].elapsed_time(ev[i + 1]) * 1e3 for i in range(args.reps)]
+    med = float(np.median(us))
+    peak, kind = load_peaks()
+    gbs = nbytes / med / 1e3
+    print(json.dumps({"profile": "blockattn", "batch": batch, "n": n, "block": block, "hq": hq,
+                      "hkv": hkv, "head_dim": D, "bytes_moved": nbytes, "flops": flops,
+                      "us_median": round(med, 1), "achieved_gbs": round(gbs, 1),
+                      "peak_gbs": peak, "peak_kind": kind, "frac": round(gbs / peak, 3),
+                      "tflops": round(flops / med / 1e6, 2),
+                      "us": [round(u, 1) for u in us]}))
+
+
 def aggregate(rank_bytes: float, rank_seconds: float, world: int, device="cpu"):
     """Whole-job throughput of N replicas: every rank processed `rank_bytes` in
     `rank_seconds`; the job takes as long as its slowest rank.  Returns
@@ -695,7 +751,8 @@ def main():
     ap.add_argument("--impl", default="seed", choices=["seed", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=12.0)
-    ap.add_argument("--profile", choices=["draft", "verify", "tree", "head", "draftstep"],
+    ap.add_argument("--profile", choices=["draft", "verify", "tree", "head", "draftstep",
+                                          "blockattn"],
                     default=None,
                     help="launch one attention kind a few times for an ncu capture")
     ap.add_argument("--reps", type=int, default=3)
