@@ -401,50 +401,78 @@ __device__ __noinline__ void unit_epilogue(const AttnTcParams& p, int b, int g, 
   }
 }
 
-// Merge of the pieces of pair (b, g) = (blockIdx.x / hkv, blockIdx.x % hkv)
-// when the pair's tiles span several CTAs of the attention kernel: the
-// pieces' records are combined with weights 2^(lse_i - M) / sum, in range
-// order.  One warp per query row (rows 8 * blockIdx.y + warp), one lane per 4
-// head dims; each lane reads every piece's log2-sum-exp and values in one
-// online pass, kMergeBatch pieces at a time.  Pairs that one CTA finished
-// alone return at once.
+// Merge of the pieces of a pair (b, g) whose tiles span several CTAs of the
+// attention kernel: the pieces' records are combined with weights
+// 2^(lse_i - M) / sum, in range order.  Block x looks at the boundary where
+// CTA x + 1's range starts and merges the pair that boundary splits, if it is
+// the pair's first such boundary; so the grid has one block column per
+// boundary, whatever the number of pairs.  One warp per query row (rows
+// 8 * blockIdx.y + warp), one lane per 4 head dims; each lane reads every
+// piece's log2-sum-exp and values in one online pass, kMergeBatch pieces at a
+// time.
 constexpr int kMergeThreads = 256;
 constexpr int kMergeRows = kMergeThreads / 32;
 constexpr int kMergeBatch = 8;
 
 __global__ void __launch_bounds__(kMergeThreads) attn_merge_kernel(const AttnTcParams p) {
-  __shared__ long long red[2][kMergeRows];
+  __shared__ long long sh_pc;
+  __shared__ int sh_b, sh_g;
   if (threadIdx.x == 0) pdl_trigger();
   pdl_wait();
-  const int pair = blockIdx.x;
-  const int b = pair / p.hkv, g = pair - b * p.hkv;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  long long tot = 0, pre = 0;
-  for (int i = tid; i < p.B; i += kMergeThreads) {
-    const long long c = seq_cost(p, seq_of(p, i).tiles);
-    tot += c;
-    if (i < b) pre += c;
+  // Block x handles range boundary c = x + 1 (the first unit of CTA c): the
+  // pair whose tiles that boundary splits, if any, and only when it is the
+  // first boundary inside the pair (CTA c - 1 holds the pair's first tile);
+  // so every shared pair is merged once and unshared pairs cost nothing.
+  const int c = blockIdx.x + 1;
+  // the cost line, block-parallel: thread i sums a contiguous chunk of
+  // sequences, a scan of the chunk sums gives T and each chunk's first unit,
+  // and the thread whose chunk holds unit x = start(c) walks it
+  __shared__ long long csum[kMergeThreads];
+  const int ch = (p.B + kMergeThreads - 1) / kMergeThreads;
+  const int b0 = tid * ch, b1 = min(p.B, b0 + ch);
+  long long mine = 0;
+  for (int i = b0; i < b1; ++i) mine += seq_cost(p, seq_of(p, i).tiles);
+  csum[tid] = mine;
+  if (tid == 0) sh_b = p.B;
+  __syncthreads();
+  for (int o = 1; o < kMergeThreads; o <<= 1) {   // inclusive scan
+    const long long v = tid >= o ? csum[tid - o] : 0;
+    __syncthreads();
+    csum[tid] += v;
+    __syncthreads();
   }
-  for (int o = 16; o; o >>= 1) {
-    tot += __shfl_xor_sync(kFull, tot, o);
-    pre += __shfl_xor_sync(kFull, pre, o);
-  }
-  if (lane == 0) {
-    red[0][warp] = tot;
-    red[1][warp] = pre;
+  const long long T = csum[kMergeThreads - 1];
+  const long long x = range_start(T, c, p.nctas);
+  long long base = csum[tid] - mine;
+  if (x < T && base <= x && x < csum[tid] && mine > 0) {
+    for (int i = b0; i < b1; ++i) {
+      const int tiles = seq_of(p, i).tiles;
+      const long long a = seq_cost(p, tiles);
+      if (x < base + a) {
+        const int per = tiles + kPairCost;
+        const int gg = (int)((x - base) / per);
+        const long long pc = base + (long long)gg * per;
+        const long long u0 = pc + kPairCost;
+        // the boundary splits the pair's tiles (x after its first tile) and
+        // is the first boundary to do so (CTA c - 1 holds the first tile)
+        if (x > u0 && cta_of(u0, T, p.nctas) == c - 1) {
+          sh_b = i;
+          sh_g = gg;
+          sh_pc = pc;
+        }
+        break;
+      }
+      base += a;
+    }
   }
   __syncthreads();
-  tot = pre = 0;
-#pragma unroll
-  for (int w = 0; w < kMergeRows; ++w) {
-    tot += red[0][w];
-    pre += red[1][w];
-  }
+  const int b = sh_b, g = sh_g;
+  if (b >= p.B) return;
   const SeqT sq = seq_of(p, b);
   const int r = blockIdx.y * kMergeRows + warp;   // query row j * G + head
   if (sq.tiles == 0 || r >= sq.nq * p.G) return;
-  const long long T = tot;
-  const long long pc = pre + (long long)g * (sq.tiles + kPairCost);   // the pair's first unit
+  const long long pc = sh_pc;                      // the pair's first unit
   const long long u0 = pc + kPairCost, u1 = u0 + sq.tiles - 1;         // its first and last tile
   const int c_lo = cta_of(u0, T, p.nctas), c_hi = cta_of(u1, T, p.nctas);
   if (c_lo == c_hi) return;
@@ -1109,7 +1137,8 @@ cudaError_t launch_attn_tc(const AttnTcParams& prm, const void* q, const void* k
   e = launch_pdl(attn_tc_kernel, dim3(prm.nctas), dim3(kThreadsTC), kSmemTC, st, tq, pm, tdk, tdv,
                  prm);
   if (e != cudaSuccess) return e;
-  const dim3 mgrid(prm.B * prm.hkv, (prm.G * prm.W1 + kMergeRows - 1) / kMergeRows);
+  if (prm.nctas < 2) return cudaSuccess;        // one CTA: no pair is shared
+  const dim3 mgrid(prm.nctas - 1, (prm.G * prm.W1 + kMergeRows - 1) / kMergeRows);
   return launch_pdl(attn_merge_kernel, mgrid, dim3(kMergeThreads), 0, st, prm);
 }
 
