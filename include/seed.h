@@ -390,9 +390,9 @@ size_t seed_draft_layer_workspace_bytes(const seed_cfg_t* cfg, const seed_decode
  *   draft_lens int32 [batch]: i after this step (1..kmax); 0 skips the
  *              sequence (its x row is then unspecified)
  * The step's token sits at position L + i - 1.  Launches norm, QKV product,
- * q/k norm + RoPE, draft KV append, draft attention, output product with
- * residual, norm, gate/up product with SwiGLU and down product with residual,
- * in this order on `stream`.
+ * q/k norm + RoPE (which writes the step's K/V row into the draft scratch),
+ * draft attention, output product with residual, norm, gate/up product with
+ * SwiGLU and down product with residual, in this order on `stream`.
  * Errors: as seed_draft_attn and seed_linear.  Device errors: as
  * seed_draft_attn, plus SEED_DEVERR_TIMEOUT. */
 seed_status_t seed_draft_layer(const seed_cfg_t* cfg, int32_t batch,

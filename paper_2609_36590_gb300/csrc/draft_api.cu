@@ -25,7 +25,7 @@ bool linear_shape_ok(int32_t batch, int32_t n_out, int32_t k_in, int32_t epi) {
 
 // The layer's temporaries, carved from its workspace.
 struct LayerWs {
-  size_t attn, lin, a, qkv, q, k, v, o, ob, m, act, total;
+  size_t attn, lin, a, qkv, q, o, ob, m, act, total;
 };
 
 LayerWs layer_ws(const seed_cfg_t* cfg, const seed_decoder_layer_t* L, int32_t B) {
@@ -47,8 +47,6 @@ LayerWs layer_ws(const seed_cfg_t* cfg, const seed_decoder_layer_t* L, int32_t B
   w.a = take((size_t)B * L->d_model * 2);
   w.qkv = take((size_t)B * nqkv * 4);
   w.q = take((size_t)B * hq * D * 2);
-  w.k = take((size_t)B * hkv * D * 2);
-  w.v = take((size_t)B * hkv * D * 2);
   w.o = take((size_t)B * hq * D * 4);
   w.ob = take((size_t)B * hq * D * 2);
   w.m = take((size_t)B * L->d_model * 2);
@@ -154,12 +152,12 @@ seed_status_t seed_draft_layer(const seed_cfg_t* cfg, int32_t batch,
   if ((s = seed_linear(batch, dm, nqkv, at(w.a), L.w_qkv, nullptr, SEED_LINEAR_F32, at(w.qkv),
                        at(w.lin), lin_bytes, err_flag, stream)) != SEED_OK)
     return s;
+  // q/k norms and RoPE; k and v land in row i-1 of the draft scratch (the
+  // draft KV append of this step)
   if ((s = fin(seedk::launch_qk_norm_rope(
            batch, hq, hkv, D, static_cast<const float*>(at(w.qkv)), L.g_q, L.g_k, ctx_lens,
-           draft_lens, L.rope_theta, L.rms_eps, at(w.q), at(w.k), at(w.v), st))) != SEED_OK)
-    return s;
-  if ((s = seed_draft_kv_append(cfg, batch, at(w.k), at(w.v), draft_lens, draft_k, draft_v,
-                                err_flag, stream)) != SEED_OK)
+           draft_lens, L.rope_theta, L.rms_eps, cfg->kmax, at(w.q), draft_k, draft_v, err_flag,
+           st))) != SEED_OK)
     return s;
   if ((s = seed_draft_attn(cfg, batch, at(w.q), ctx_kv, draft_k, draft_v, ctx_lens, draft_lens,
                            static_cast<float*>(at(w.o)), nullptr, at(w.attn),

@@ -102,7 +102,9 @@ __global__ void __launch_bounds__(kOpsThreads) rmsnorm_kernel(int32_t n, const f
 
 // From qkv f32 [B, (hq + 2 hkv) D]: q, k normed per head (gain g_q / g_k) and
 // rotated (rotate-half pairs (i, i + D/2), angle pos * theta^(-2i/D)); v
-// copied; all three rounded to bf16.  pos = ctx_len + draft_len - 1: the
+// copied; all three rounded to bf16.  q goes to q [B, hq, D]; k and v go
+// straight to row draft_len - 1 of the layer's draft scratch [B, hkv, kmax,
+// D] (the draft KV append of this step).  pos = ctx_len + draft_len - 1: the
 // position of the token this draft step feeds.  One warp per (sequence,
 // head).  The frequencies theta^(-2i/D) come from the host in double; each
 // lane forms its angle pos * w in double and reduces it by 2 pi (split in two
@@ -115,7 +117,8 @@ struct RopeFreq {
 __global__ void __launch_bounds__(kRopeWarps * 32) qk_norm_rope_kernel(
     int32_t hq, int32_t hkv, int32_t D, const float* qkv, const __nv_bfloat16* gq,
     const __nv_bfloat16* gk, const int32_t* ctx_lens, const int32_t* draft_lens,
-    const RopeFreq fr, float eps, __nv_bfloat16* q, __nv_bfloat16* k, __nv_bfloat16* v) {
+    const RopeFreq fr, float eps, int32_t kmax, __nv_bfloat16* q, __nv_bfloat16* dk,
+    __nv_bfloat16* dv, int32_t* err) {
   if (threadIdx.x == 0) pdl_trigger();
   pdl_wait();
   const int b = blockIdx.x;
@@ -125,16 +128,21 @@ __global__ void __launch_bounds__(kRopeWarps * 32) qk_norm_rope_kernel(
   if (h >= nh) return;
   const int dl = draft_lens[b];
   if (dl <= 0) return;                        // skipped sequence
+  if (dl > kmax) {
+    if (lane == 0) raise_err(err, SEED_DEVERR_DRAFT_LEN);
+    return;
+  }
   const float* xh = qkv + ((size_t)b * nh + h) * D;
   const int half = D / 2;                     // 32 or 64: one or two pairs per lane
   if (h >= hq + hkv) {                        // v: copy
-    __nv_bfloat16* dst = v + ((size_t)b * hkv + (h - hq - hkv)) * D;
+    __nv_bfloat16* dst = dv + (((size_t)b * hkv + (h - hq - hkv)) * kmax + dl - 1) * D;
     for (int i = lane; i < D; i += 32) dst[i] = __float2bfloat16_rn(xh[i]);
     return;
   }
   const bool isq = h < hq;
   const __nv_bfloat16* g = isq ? gq : gk;
-  __nv_bfloat16* dst = isq ? q + ((size_t)b * hq + h) * D : k + ((size_t)b * hkv + (h - hq)) * D;
+  __nv_bfloat16* dst = isq ? q + ((size_t)b * hq + h) * D
+                            : dk + (((size_t)b * hkv + (h - hq)) * kmax + dl - 1) * D;
   const int np = half / 32;                   // pairs per lane
   float a[2], c[2];
   float ss = 0.f;
@@ -194,15 +202,16 @@ cudaError_t launch_rmsnorm(int32_t rows, int32_t n, const float* x, const void* 
 
 cudaError_t launch_qk_norm_rope(int32_t B, int32_t hq, int32_t hkv, int32_t D, const float* qkv,
                                 const void* gq, const void* gk, const int32_t* ctx_lens,
-                                const int32_t* draft_lens, float theta, float eps, void* q,
-                                void* k, void* v, cudaStream_t st) {
+                                const int32_t* draft_lens, float theta, float eps, int32_t kmax,
+                                void* q, void* draft_k, void* draft_v, int32_t* err,
+                                cudaStream_t st) {
   RopeFreq fr{};
   for (int i = 0; i < D / 2 && i < 64; ++i) fr.w[i] = std::pow((double)theta, -2.0 * i / D);
   const dim3 grid(B, (hq + 2 * hkv + kRopeWarps - 1) / kRopeWarps);
   return launch_pdl(qk_norm_rope_kernel, grid, dim3(kRopeWarps * 32), 0, st, hq, hkv, D, qkv,
                     static_cast<const __nv_bfloat16*>(gq), static_cast<const __nv_bfloat16*>(gk),
-                    ctx_lens, draft_lens, fr, eps, static_cast<__nv_bfloat16*>(q),
-                    static_cast<__nv_bfloat16*>(k), static_cast<__nv_bfloat16*>(v));
+                    ctx_lens, draft_lens, fr, eps, kmax, static_cast<__nv_bfloat16*>(q),
+                    static_cast<__nv_bfloat16*>(draft_k), static_cast<__nv_bfloat16*>(draft_v), err);
 }
 
 cudaError_t launch_f32_to_bf16(size_t n, const float* x, void* y, cudaStream_t st) {

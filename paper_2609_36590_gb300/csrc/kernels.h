@@ -143,8 +143,9 @@ cudaError_t launch_rmsnorm(int32_t rows, int32_t n, const float* x, const void* 
                            void* y, cudaStream_t st);
 cudaError_t launch_qk_norm_rope(int32_t B, int32_t hq, int32_t hkv, int32_t D, const float* qkv,
                                 const void* gq, const void* gk, const int32_t* ctx_lens,
-                                const int32_t* draft_lens, float theta, float eps, void* q,
-                                void* k, void* v, cudaStream_t st);
+                                const int32_t* draft_lens, float theta, float eps, int32_t kmax,
+                                void* q, void* draft_k, void* draft_v, int32_t* err,
+                                cudaStream_t st);
 cudaError_t launch_f32_to_bf16(size_t n, const float* x, void* y, cudaStream_t st);
 
 // Tensor-core draft and verify attention (attn_tc.cu).
