@@ -81,10 +81,10 @@ def round_bytes(wl, lens: np.ndarray, k_b: np.ndarray, n_layers: int) -> dict:
 # reported traffic is scaled to the timed launches by their algorithmic bytes,
 # and is null once the kernel's sources differ from the captured ones.
 NCU_TRAFFIC = {
-    (4, "verify"): {"kernel": "attn_tc_kernel", "sources": "9e062419c2dd7da4",
-                    "dram_bytes": 538029056 + 10626048, "alg_bytes": 537907712},
-    (4, "draft"): {"kernel": "attn_tc_kernel", "sources": "9e062419c2dd7da4",
-                   "dram_bytes": 537450496 + 10451968, "alg_bytes": 536986112},
+    (4, "verify"): {"kernel": "attn_tc_kernel", "sources": "e62147c3b201117d",
+                    "dram_bytes": 538025728 + 10420480, "alg_bytes": 537907712},
+    (4, "draft"): {"kernel": "attn_tc_kernel", "sources": "e62147c3b201117d",
+                   "dram_bytes": 537406720 + 10487040, "alg_bytes": 536986112},
 }
 
 KERNEL_SOURCES = {
