@@ -46,6 +46,16 @@ def load_peaks():
     return 6800.0, "fallback"
 
 
+def load_bf16_peak():
+    """Dense bf16 tensor-core peak (TFLOP/s, burst) from the measured file, else
+    the fallback figure."""
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            return float(json.load(f)["bf16_tflops"])
+    return 1900.0
+
+
 # ------------------------------------------------------------------ accounting
 def round_bytes(wl, lens: np.ndarray, k_b: np.ndarray, n_layers: int) -> dict:
     """Algorithmic bytes of one round.  R = K+V bytes of one token in one layer.
@@ -615,22 +625,30 @@ def run_profile_blockattn(args, wl, n=1000, block=10, batch=8):
     assert int(err.item()) == 0, "device error flag raised"
     R = 2 * hkv * D * 2                               # K + V bytes of one row
     nblk = n // block
-    rows_read = sum(s * block + block for s in range(nblk))      # deep prefix + own rows
-    pages = -(-n // 16) + nblk * -(-(15 + block) // 16)
-    copy = (n * 2 * R) + pages * 16 * R               # read 4 inputs, write the paged copy
     qo = n * hq * (D * (2 + 4) + 4)
-    nbytes = batch * (rows_read * R + pages * 16 * R + copy + qo)
+    if D == 128 and hq // hkv in (1, 2, 4):
+        # tensor-core route: every input read once, o and lse written once
+        route = "tensor-core"
+        nbytes = batch * (2 * n * R + qo)
+    else:
+        route = "virtual-sequence"
+        rows_read = sum(s * block + block for s in range(nblk))  # deep prefix + own rows
+        pages = -(-n // 16) + nblk * -(-(15 + block) // 16)
+        copy = (n * 2 * R) + pages * 16 * R           # read 4 inputs, write the paged copy
+        nbytes = batch * (rows_read * R + pages * 16 * R + copy + qo)
     vis = sum(s * block + (j + 1) for s in range(nblk) for j in range(block))
     flops = batch * hq * vis * D * 4
     us = [ev[i].elapsed_time(ev[i + 1]) * 1e3 for i in range(args.reps)]
     med = float(np.median(us))
     peak, kind = load_peaks()
     gbs = nbytes / med / 1e3
-    print(json.dumps({"profile": "blockattn", "batch": batch, "n": n, "block": block, "hq": hq,
+    print(json.dumps({"profile": "blockattn", "route": route, "batch": batch, "n": n,
+                      "block": block, "hq": hq,
                       "hkv": hkv, "head_dim": D, "bytes_moved": nbytes, "flops": flops,
                       "us_median": round(med, 1), "achieved_gbs": round(gbs, 1),
                       "peak_gbs": peak, "peak_kind": kind, "frac": round(gbs / peak, 3),
                       "tflops": round(flops / med / 1e6, 2),
+                      "bf16_peak_tflops": load_bf16_peak(),
                       "us": [round(u, 1) for u in us]}))
 
 

@@ -21,7 +21,7 @@ LIB = os.path.join(PKG, "libseed.so")
 
 SOURCES = ["seed_api.cu", "decode_attn.cu", "cache_accept.cu", "attn_tc.cu", "noalloc_api.cu",
            "head_tc.cu", "linear_tc.cu", "draft_ops.cu", "draft_api.cu",
-           "block_attn.cu"]
+           "block_attn.cu", "block_tc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
          "--expt-relaxed-constexpr", "-I", os.path.join(ROOT, "include")]

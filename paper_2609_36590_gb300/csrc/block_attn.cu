@@ -15,17 +15,28 @@
 // on all blocks at once: q [batch, n, hq, D] is already the virtual batch's
 // [batch * n/b, b, hq, D] layout, and so are out and lse.
 //
-// Cost: each block reads its deep prefix again (about n^2 / 2b rows per
-// sequence and KV head instead of a prefill kernel's n^2 / 2 x 128 rows), so
-// the call is bound by HBM rather than by the tensor cores.
+// head_dim 128 with groups of 1, 2 or 4 query heads per KV head goes to the
+// prefill-style tensor-core kernel of block_tc.cu instead, which reads each
+// query tile's prefix once for 128 query rows; the virtual-sequence route
+// (which re-reads each block's prefix, about n^2 / 2b rows per sequence and
+// KV head) serves the other shapes.
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <cmath>
 #include <cstdint>
 
 #include "../../include/seed.h"
 #include "common.cuh"
 #include "kernels.h"
+
+namespace seedk {
+bool block_tc_supported(int32_t head_dim, int32_t group);
+cudaError_t launch_block_tc(int32_t B, int32_t n, int32_t blk, int32_t hq, int32_t hkv,
+                            float scale, const void* q, const void* k_dec, const void* v_dec,
+                            const void* k_spec, const void* v_spec, float* out, float* lse,
+                            int32_t* err, cudaStream_t st);
+}  // namespace seedk
 
 namespace {
 
@@ -175,6 +186,7 @@ extern "C" {
 size_t seed_block_attn_workspace_bytes(const seed_cfg_t* cfg, int32_t batch, int32_t n,
                                        int32_t block) {
   if (!block_ok(cfg, batch, n, block) || batch == 0) return 0;
+  if (seedk::block_tc_supported(cfg->head_dim, cfg->hq / cfg->hkv)) return 256;   // unused
   const BlockGeom g = geom(batch, n, block, cfg->hkv, cfg->head_dim);
   if (g.num_pages > INT32_MAX) return 0;
   const seed_cfg_t v = virtual_cfg(cfg, block);
@@ -193,6 +205,14 @@ seed_status_t seed_block_attn(const seed_cfg_t* cfg, int32_t batch, int32_t n, i
   auto mis16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) != 0; };
   if (mis16(q) || mis16(k_dec) || mis16(v_dec) || mis16(k_spec) || mis16(v_spec) || mis16(out))
     return SEED_ERR_RANGE;
+  if (seedk::block_tc_supported(cfg->head_dim, cfg->hq / cfg->hkv)) {
+    if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0 || ws_bytes < 256) return SEED_ERR_WORKSPACE;
+    const float scale = cfg->scale > 0.f ? cfg->scale : 1.0f / std::sqrt((float)cfg->head_dim);
+    const cudaError_t e = seedk::launch_block_tc(batch, n, block, cfg->hq, cfg->hkv, scale, q,
+                                                 k_dec, v_dec, k_spec, v_spec, out, lse,
+                                                 err_flag, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? SEED_OK : SEED_ERR_CUDA;
+  }
   const BlockGeom g = geom(batch, n, block, cfg->hkv, cfg->head_dim);
   if (g.num_pages > INT32_MAX) return SEED_ERR_SHAPE;
   const seed_cfg_t v = virtual_cfg(cfg, block);

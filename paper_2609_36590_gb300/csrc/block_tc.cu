@@ -1,0 +1,500 @@
+// Block-causal training attention on the tensor cores (Sec. 3, "Training
+// with Block Attention"; Fig. 2): the query at position p sees the deep rows
+// KV^dec at positions < s(p) = (p / b) * b and its own block's raw-embedding
+// rows at positions s(p) .. p.
+//
+// A prefill-style kernel for head_dim 128: each CTA takes 128 query rows --
+// 128 / G consecutive positions times the G query heads of one KV head, the
+// row of (position i, head j) being i * G + j -- and streams the key tiles it
+// needs once: the deep rows below the tile's last block start, then the raw-
+// embedding rows from its first block start to its last position.  Per tile,
+// S = Q K^T (tcgen05, bf16 -> f32 in TMEM), an online softmax in the log2
+// domain with the block mask, and O += P V with P split into bf16 hi + lo
+// terms (so P carries 16 significant bits).  Two S/P buffers let S(t+1) run
+// while tile t's softmax runs.
+//
+// Warp roles (320 threads): warps 0-7 softmax and epilogue -- warp w takes
+// TMEM lane quarter w % 4 and key / output columns [64 (w / 4), + 64), the
+// two halves of a row trading their maxima through shared memory -- warp 8
+// TMA producer, warp 9 MMA issuer and TMEM owner.
+// Every wait is bounded; a wait that gives up raises SEED_DEVERR_TIMEOUT, and
+// the CTA still drains its copies and MMAs before it frees TMEM and exits.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <atomic>
+#include <cmath>
+#include <mutex>
+
+#include "common.cuh"
+#include "kernels.h"
+#include "tc.cuh"
+
+namespace seedk {
+namespace {
+
+constexpr int kBD = 128;                       // head_dim
+constexpr int kBN = 128;                       // keys per tile
+constexpr int kBThreads = 320;
+constexpr int kBSoftWarps = 8;
+constexpr int kBWarpProd = 8, kBWarpMma = 9;
+constexpr uint32_t kBHalf = 128 * 128;         // 128 rows x 128 B
+constexpr uint32_t kBTile = 2 * kBHalf;        // one tile of Q, K or V: two head-dim halves
+constexpr uint32_t kBOffK = kBTile;            // Q at 0, then the K ring, then the V ring
+constexpr uint32_t kBOffV = kBOffK + 2 * kBTile;
+constexpr uint32_t kBOffCtrl = kBOffV + 2 * kBTile;
+constexpr uint32_t kBOffX = kBOffCtrl + 256;   // f32 [2 tiles][2 halves][128 rows] row maxima
+constexpr uint32_t kBOffL = kBOffX + 2048;     // f32 [2 halves][128 rows] row sums
+constexpr uint32_t kBColO = 256;               // S/P buffers [0, 256), O [256, 384)
+constexpr uint32_t kBIdescS = idesc_bf16_f32(128, kBN, 0, 0);   // K-major A and B
+constexpr uint32_t kBIdescPV = idesc_bf16_f32(128, kBD, 0, 1);  // B (V) MN-major
+constexpr float kBRescale = 8.0f;
+constexpr float kBLn2 = 0.69314718055994531f;
+constexpr unsigned kBFull = 0xffffffffu;
+
+struct BCtrl {
+  uint64_t q_full;
+  uint64_t k_full[2], k_empty[2], v_full[2], v_empty[2];
+  uint64_t s_full[2], p_full[2];
+  uint64_t x_full[2], l_full;                  // the softmax warps' exchanges
+  uint64_t o_full, mma_done;
+  uint32_t tmem_base;
+  volatile int32_t abort_flag;
+};
+constexpr size_t kBSmem = kBOffL + 1024 + 1024;
+static_assert(sizeof(BCtrl) <= 256, "control block");
+
+struct BlockTcParams {
+  float* out;          // f32 [B, n, hq, D]
+  float* lse;          // f32 [B, n, hq] or null
+  int32_t* err;
+  int32_t B, n, blk, hq, hkv, G, P, nqt;
+  float c2;            // softmax scale * log2(e)
+};
+
+__device__ __noinline__ bool bwait(uint64_t* bar, uint32_t parity, BCtrl* c, int32_t* err) {
+  for (uint32_t i = 0; i < kSuspendTries; ++i) {
+    if (mbar_try_wait_sleep(bar, parity, kSuspendNs)) return true;
+    if (c->abort_flag) return false;
+  }
+  c->abort_flag = 1;
+  raise_err(err, SEED_DEVERR_TIMEOUT);
+  return false;
+}
+
+__device__ __forceinline__ bool bwarp_wait(uint64_t* bar, uint32_t parity, BCtrl* c,
+                                           int32_t* err) {
+  return __all_sync(kBFull, bwait(bar, parity, c, err));
+}
+
+__device__ __forceinline__ bool bpoll(uint64_t* bar, uint32_t parity, BCtrl* c, int32_t* err) {
+  for (uint32_t i = 0; i < (1u << 26); ++i) {
+    if (mbar_test(bar, parity)) return true;
+    if ((i & 1023u) == 1023u && c->abort_flag) return false;
+  }
+  c->abort_flag = 1;
+  raise_err(err, SEED_DEVERR_TIMEOUT);
+  return false;
+}
+
+__device__ __forceinline__ void bdrain(uint64_t* bar, uint32_t parity, int32_t* err) {
+  for (uint32_t i = 0; i < (1u << 26); ++i)
+    if (mbar_test(bar, parity)) return;
+  raise_err(err, SEED_DEVERR_TIMEOUT);
+}
+
+// Bits of the 32 keys k0 .. k0 + 31 that lie in [lo, hi].
+__device__ __forceinline__ uint32_t key_bits(int k0, int lo, int hi) {
+  const int a = max(lo - k0, 0), e = min(hi - k0, 31);
+  if (e < a) return 0u;
+  const uint32_t w = (uint32_t)(e - a + 1);
+  return (w == 32u ? 0xffffffffu : ((1u << w) - 1u)) << a;
+}
+
+// The CTA's query tile and its key tiles.
+struct BTiles {
+  int b, g, p0, plast, s_lo, nd, nt;
+};
+
+__device__ __forceinline__ BTiles tiles_of(const BlockTcParams& p) {
+  BTiles t;
+  const int per = p.B * p.hkv;
+  const int qt = p.nqt - 1 - (int)(blockIdx.x / per);   // longest prefixes first
+  const int rest = (int)(blockIdx.x % per);
+  t.b = rest / p.hkv;
+  t.g = rest - t.b * p.hkv;
+  t.p0 = qt * p.P;
+  t.plast = min(t.p0 + p.P, p.n) - 1;
+  t.s_lo = (t.p0 / p.blk) * p.blk;
+  const int s_hi = (t.plast / p.blk) * p.blk;
+  t.nd = (s_hi + kBN - 1) / kBN;                          // deep tiles: rows [0, s_hi)
+  t.nt = t.nd + (t.plast + 1 - t.s_lo + kBN - 1) / kBN;   // then rows [s_lo, plast]
+  return t;
+}
+
+__global__ void __launch_bounds__(kBThreads, 1) block_tc_kernel(
+    const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kd,
+    const __grid_constant__ CUtensorMap tm_vd, const __grid_constant__ CUtensorMap tm_ks,
+    const __grid_constant__ CUtensorMap tm_vs, const BlockTcParams p) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+  BCtrl* ctrl = reinterpret_cast<BCtrl*>(smem + kBOffCtrl);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const uint32_t sbase = smem_u32(smem);
+  if (tid == 0) pdl_trigger();
+  if (tid == 0) {
+    mbar_init(&ctrl->q_full, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&ctrl->k_full[i], 1);
+      mbar_init(&ctrl->k_empty[i], 1);
+      mbar_init(&ctrl->v_full[i], 1);
+      mbar_init(&ctrl->v_empty[i], 1);
+      mbar_init(&ctrl->s_full[i], 1);
+      mbar_init(&ctrl->p_full[i], kBSoftWarps);
+      mbar_init(&ctrl->x_full[i], kBSoftWarps);
+    }
+    mbar_init(&ctrl->l_full, kBSoftWarps);
+    mbar_init(&ctrl->o_full, 1);
+    mbar_init(&ctrl->mma_done, 1);
+    ctrl->abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == kBWarpMma) {
+    tmem_alloc(&ctrl->tmem_base, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = ctrl->tmem_base;
+  pdl_wait();
+  const BTiles T = tiles_of(p);
+
+  if (warp == kBWarpProd) {
+    // ---------------------------------------------------------- TMA producer
+    if (lane == 0) {
+      tma_prefetch_desc(&tm_q);
+      tma_prefetch_desc(&tm_kd);
+      tma_prefetch_desc(&tm_vd);
+      tma_prefetch_desc(&tm_ks);
+      tma_prefetch_desc(&tm_vs);
+      mbar_arrive_expect_tx(&ctrl->q_full, kBTile);
+      tma_load_4d(smem, &tm_q, 0, T.g * p.G, T.p0, T.b, &ctrl->q_full);
+      tma_load_4d(smem + kBHalf, &tm_q, 64, T.g * p.G, T.p0, T.b, &ctrl->q_full);
+      int kiss = 0, viss = 0;                  // K and V tiles issued
+      for (int t = 0; t < T.nt; ++t) {
+        const int s = t & 1;
+        const uint32_t ph = (uint32_t)(((t >> 1) - 1) & 1);
+        const bool deep = t < T.nd;
+        const int k0 = deep ? t * kBN : T.s_lo + (t - T.nd) * kBN;
+        const CUtensorMap* mk = deep ? &tm_kd : &tm_ks;
+        const CUtensorMap* mv = deep ? &tm_vd : &tm_vs;
+        if (t >= 2 && !bpoll(&ctrl->k_empty[s], ph, ctrl, p.err)) break;
+        uint8_t* kb = smem + kBOffK + s * kBTile;
+        mbar_arrive_expect_tx(&ctrl->k_full[s], kBTile);
+        tma_load_4d(kb, mk, 0, T.g, k0, T.b, &ctrl->k_full[s]);
+        tma_load_4d(kb + kBHalf, mk, 64, T.g, k0, T.b, &ctrl->k_full[s]);
+        ++kiss;
+        if (t >= 2 && !bpoll(&ctrl->v_empty[s], ph, ctrl, p.err)) break;
+        uint8_t* vb = smem + kBOffV + s * kBTile;
+        mbar_arrive_expect_tx(&ctrl->v_full[s], kBTile);
+        tma_load_4d(vb, mv, 0, T.g, k0, T.b, &ctrl->v_full[s]);
+        tma_load_4d(vb + kBHalf, mv, 64, T.g, k0, T.b, &ctrl->v_full[s]);
+        ++viss;
+      }
+      // every copy this CTA started has landed before it moves on (the last
+      // fill of each ring slot; earlier fills were consumed before reuse)
+      bdrain(&ctrl->q_full, 0, p.err);
+      for (int j = max(0, kiss - 2); j < kiss; ++j)
+        bdrain(&ctrl->k_full[j & 1], (uint32_t)((j >> 1) & 1), p.err);
+      for (int j = max(0, viss - 2); j < viss; ++j)
+        bdrain(&ctrl->v_full[j & 1], (uint32_t)((j >> 1) & 1), p.err);
+    }
+    __syncwarp();
+  } else if (warp == kBWarpMma) {
+    // ---------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      int ts = 0, tp = 0;
+      bool ok = bpoll(&ctrl->q_full, 0, ctrl, p.err);
+      uint32_t idle = 0;
+      while (ok && tp < T.nt && !ctrl->abort_flag) {
+        bool did = false;
+        if (ts < T.nt && ts <= tp + 1 &&
+            mbar_test(&ctrl->k_full[ts & 1], (uint32_t)((ts >> 1) & 1))) {
+          tc_fence_after();
+          const uint32_t d = tmem + (uint32_t)(ts & 1) * kBN;
+          const uint32_t kb = sbase + kBOffK + (uint32_t)(ts & 1) * kBTile;
+#pragma unroll
+          for (int kk = 0; kk < kBD / 16; ++kk) {
+            const uint32_t h = kk >> 2, off = (kk & 3) * 32;
+            const uint64_t a = smem_desc_sw128(sbase + h * kBHalf + off, 16, 1024);
+            const uint64_t bd = smem_desc_sw128(kb + h * kBHalf + off, 16, 1024);
+            mma_ss(d, a, bd, kBIdescS, kk > 0 ? 1u : 0u);
+          }
+          mma_commit(&ctrl->s_full[ts & 1]);
+          mma_commit(&ctrl->k_empty[ts & 1]);
+          ++ts;
+          did = true;
+        }
+        if (tp < ts && mbar_test(&ctrl->p_full[tp & 1], (uint32_t)((tp >> 1) & 1)) &&
+            mbar_test(&ctrl->v_full[tp & 1], (uint32_t)((tp >> 1) & 1))) {
+          tc_fence_after();
+          const uint32_t pcol = tmem + (uint32_t)(tp & 1) * kBN;
+          const uint32_t ocol = tmem + kBColO;
+          const uint32_t vb = sbase + kBOffV + (uint32_t)(tp & 1) * kBTile;
+          // keys [16 kk, 16 kk + 16): P_hi at packed column 32 (kk / 2) + 8 (kk % 2),
+          // P_lo 16 columns further
+#pragma unroll
+          for (int kk = 0; kk < kBN / 16; ++kk) {
+            const uint64_t bd = smem_desc_sw128(vb + kk * 2048u, kBHalf, 1024);
+            const uint32_t a = pcol + 32 * (kk >> 1) + 8 * (kk & 1);
+            mma_ts(ocol, a, bd, kBIdescPV, (tp > 0 || kk > 0) ? 1u : 0u);
+            mma_ts(ocol, a + 16, bd, kBIdescPV, 1u);
+          }
+          mma_commit(&ctrl->o_full);
+          mma_commit(&ctrl->v_empty[tp & 1]);
+          ++tp;
+          did = true;
+        }
+        if (did) {
+          idle = 0;
+        } else if (++idle > (1u << 28)) {
+          ctrl->abort_flag = 1;
+          raise_err(p.err, SEED_DEVERR_TIMEOUT);
+        }
+      }
+      mma_commit(&ctrl->mma_done);
+      bdrain(&ctrl->mma_done, 0, p.err);
+    }
+    __syncwarp();
+  } else {
+    // ---------------------------------------------------------- softmax + epilogue
+    const int q4 = warp & 3, hf = warp >> 2;  // lane quarter, column half
+    const int row = q4 * 32 + lane;
+    const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
+    float* xs = reinterpret_cast<float*>(smem + kBOffX);
+    float* ls_sh = reinterpret_cast<float*>(smem + kBOffL);
+    const int pos = T.p0 + row / p.G;
+    const bool real = pos <= T.plast;
+    const int sp = (pos / p.blk) * p.blk;     // this row's block start
+    float m_used = -INFINITY, l = 0.f;
+    bool ok = true;
+    for (int t = 0; t < T.nt && ok; ++t) {
+      ok = bwarp_wait(&ctrl->s_full[t & 1], (uint32_t)((t >> 1) & 1), ctrl, p.err);
+      if (!ok) break;
+      tc_fence_after();
+      const bool deep = t < T.nd;
+      const int k0 = (deep ? t * kBN : T.s_lo + (t - T.nd) * kBN) + 64 * hf;
+      const int lo = real ? (deep ? 0 : sp) : 1;
+      const int hi = real ? (deep ? sp - 1 : pos) : 0;   // visible keys [lo, hi]
+      const uint32_t scol = tmem + lane_off + (uint32_t)(t & 1) * kBN + 64u * hf;
+      uint32_t ra[32], rb[32];
+      tmem_ld32(scol, ra);
+      tmem_ld32(scol + 32, rb);
+      tmem_wait_ld();
+      const uint32_t ba = key_bits(k0, lo, hi), bb = key_bits(k0 + 32, lo, hi);
+      float mx = -INFINITY;
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        if ((ba >> i) & 1u) mx = fmaxf(mx, __uint_as_float(ra[i]));
+        if ((bb >> i) & 1u) mx = fmaxf(mx, __uint_as_float(rb[i]));
+      }
+      // the row's maximum over both column halves
+      float* xt = xs + (t & 1) * 256;
+      xt[hf * 128 + row] = mx;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctrl->x_full[t & 1]);
+      ok = bwarp_wait(&ctrl->x_full[t & 1], (uint32_t)((t >> 1) & 1), ctrl, p.err);
+      if (!ok) break;
+      mx = fmaxf(mx, xt[(hf ^ 1) * 128 + row]);
+      const float mt = mx * p.c2;
+      bool resc = false;
+      float fo = 1.f;
+      if (mt > m_used + kBRescale) {
+        const float f = (m_used == -INFINITY) ? 0.f : ex2_approx(m_used - mt);
+        if (t > 0 && m_used != -INFINITY) {
+          resc = true;
+          fo = f;
+        }
+        l *= f;
+        m_used = mt;
+      }
+      const float mc = (m_used == -INFINITY) ? 0.f : m_used;
+      // P = 2^(s c2 - m) as bf16 hi + lo pairs, in place of S
+      float lsum = 0.f;
+      uint32_t wh[16], wl[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const float p0 = ((ba >> (2 * i)) & 1u)
+                             ? ex2_approx(fmaf(__uint_as_float(ra[2 * i]), p.c2, -mc)) : 0.f;
+        const float p1 = ((ba >> (2 * i + 1)) & 1u)
+                             ? ex2_approx(fmaf(__uint_as_float(ra[2 * i + 1]), p.c2, -mc)) : 0.f;
+        lsum += p0 + p1;
+        const uint32_t hh = pack_bf16x2(p0, p1);
+        wh[i] = hh;
+        wl[i] = pack_bf16x2(p0 - bf16lo(hh), p1 - bf16hi(hh));
+      }
+      tmem_st16(scol, wh);
+      tmem_st16(scol + 16, wl);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const float p0 = ((bb >> (2 * i)) & 1u)
+                             ? ex2_approx(fmaf(__uint_as_float(rb[2 * i]), p.c2, -mc)) : 0.f;
+        const float p1 = ((bb >> (2 * i + 1)) & 1u)
+                             ? ex2_approx(fmaf(__uint_as_float(rb[2 * i + 1]), p.c2, -mc)) : 0.f;
+        lsum += p0 + p1;
+        const uint32_t hh = pack_bf16x2(p0, p1);
+        wh[i] = hh;
+        wl[i] = pack_bf16x2(p0 - bf16lo(hh), p1 - bf16hi(hh));
+      }
+      tmem_st16(scol + 32, wh);
+      tmem_st16(scol + 48, wl);
+      tmem_wait_st();
+      l += lsum;
+      // O must be rescaled before PV(t) adds to it: wait for PV(t - 1)
+      if (__any_sync(kBFull, resc)) {
+        ok = bwarp_wait(&ctrl->o_full, (uint32_t)((t - 1) & 1), ctrl, p.err);
+        if (!ok) break;
+        tc_fence_after();
+        const uint32_t ocol = tmem + lane_off + kBColO + 64u * hf;
+#pragma unroll 1
+        for (int c = 0; c < 2; ++c) {
+          uint32_t r[32];
+          tmem_ld32(ocol + c * 32, r);
+          tmem_wait_ld();
+#pragma unroll
+          for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * fo);
+          tmem_st32(ocol + c * 32, r);
+        }
+        tmem_wait_st();
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctrl->p_full[t & 1]);
+    }
+    // epilogue: O / l once every MMA of the CTA has completed
+    if (ok) {
+      ls_sh[hf * 128 + row] = l;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctrl->l_full);
+      ok = bwarp_wait(&ctrl->l_full, 0, ctrl, p.err);
+    }
+    if (ok) {
+      l += ls_sh[(hf ^ 1) * 128 + row];
+      ok = bwarp_wait(&ctrl->mma_done, 0, ctrl, p.err);
+    }
+    if (ok) {
+      tc_fence_after();
+      const uint32_t ocol = tmem + lane_off + kBColO + 64u * hf;
+      const float inv = l > 0.f ? 1.f / l : 0.f;
+      const int h = T.g * p.G + row % p.G;
+      const size_t orow = ((size_t)T.b * p.n + (real ? pos : 0)) * p.hq + h;
+#pragma unroll 1
+      for (int c = 0; c < 4; ++c) {
+        uint32_t r[16];
+        tmem_ld16(ocol + c * 16, r);
+        tmem_wait_ld();
+        if (real) {
+          float4* dp = reinterpret_cast<float4*>(p.out + orow * kBD + 64 * hf + c * 16);
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+            dp[i] = make_float4(__uint_as_float(r[4 * i]) * inv, __uint_as_float(r[4 * i + 1]) * inv,
+                                __uint_as_float(r[4 * i + 2]) * inv,
+                                __uint_as_float(r[4 * i + 3]) * inv);
+        }
+      }
+      if (real && hf == 0 && p.lse != nullptr) p.lse[orow] = (m_used + log2f(l)) * kBLn2;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == kBWarpMma) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+// ------------------------------------------------------------- host side
+using EncodeFnB = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                               const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                               const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                               CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeFnB encode_fn_b() {
+  static EncodeFnB fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeFnB>(ptr);
+  });
+  return fn;
+}
+
+// 4-d bf16 map [B, n, heads, 128] with (64, hbox, rows, 1) boxes, 128-byte swizzle.
+bool encode_bthd(CUtensorMap* map, const void* base, int B, int n, int heads, int hbox,
+                 int rows) {
+  EncodeFnB fn = encode_fn_b();
+  if (fn == nullptr) return false;
+  const cuuint64_t dims[4] = {(cuuint64_t)kBD, (cuuint64_t)heads, (cuuint64_t)n, (cuuint64_t)B};
+  const cuuint64_t strides[3] = {(cuuint64_t)kBD * 2, (cuuint64_t)heads * kBD * 2,
+                                 (cuuint64_t)n * heads * kBD * 2};
+  const cuuint32_t box[4] = {64, (cuuint32_t)hbox, (cuuint32_t)rows, 1};
+  const cuuint32_t elem[4] = {1, 1, 1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box,
+            elem, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+std::atomic<uint64_t> g_block_attr{0};
+
+}  // namespace
+
+bool block_tc_supported(int32_t head_dim, int32_t group) {
+  return head_dim == kBD && (group == 1 || group == 2 || group == 4);
+}
+
+cudaError_t launch_block_tc(int32_t B, int32_t n, int32_t blk, int32_t hq, int32_t hkv,
+                            float scale, const void* q, const void* k_dec, const void* v_dec,
+                            const void* k_spec, const void* v_spec, float* out, float* lse,
+                            int32_t* err, cudaStream_t st) {
+  BlockTcParams p{};
+  p.out = out;
+  p.lse = lse;
+  p.err = err;
+  p.B = B;
+  p.n = n;
+  p.blk = blk;
+  p.hq = hq;
+  p.hkv = hkv;
+  p.G = hq / hkv;
+  p.P = 128 / p.G;
+  p.nqt = (n + p.P - 1) / p.P;
+  p.c2 = scale * 1.4426950408889634f;
+  CUtensorMap tq, tkd, tvd, tks, tvs;
+  if (!encode_bthd(&tq, q, B, n, hq, p.G, p.P) || !encode_bthd(&tkd, k_dec, B, n, hkv, 1, kBN) ||
+      !encode_bthd(&tvd, v_dec, B, n, hkv, 1, kBN) ||
+      !encode_bthd(&tks, k_spec, B, n, hkv, 1, kBN) ||
+      !encode_bthd(&tvs, v_spec, B, n, hkv, 1, kBN))
+    return cudaErrorInvalidValue;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const uint64_t bit = 1ull << (dev & 63);
+  if (!(g_block_attr.load(std::memory_order_acquire) & bit)) {
+    e = cudaFuncSetAttribute(block_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)kBSmem);
+    if (e != cudaSuccess) return e;
+    g_block_attr.fetch_or(bit, std::memory_order_acq_rel);
+  }
+  const long long grid = (long long)B * hkv * p.nqt;
+  if (grid <= 0 || grid > 0x7fffffffLL) return cudaErrorInvalidValue;
+  return launch_pdl(block_tc_kernel, dim3((unsigned)grid), dim3(kBThreads), kBSmem, st, tq, tkd,
+                    tvd, tks, tvs, p);
+}
+
+}  // namespace seedk

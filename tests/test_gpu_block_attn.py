@@ -2,7 +2,8 @@
 "Training with Block Attention"; Fig. 2) through the C ABI against the
 oracle: o and lse within the attention tolerance (max abs <= 2e-3, max rel
 <= 1e-2 on |o| > 1e-2) for block sizes 2 to 32, head_dim 64 and 128, group
-sizes 1 to 4, block boundaries inside and across 16-row pages; a 4B-shaped
+sizes 1 to 4, block boundaries inside and across 16-row pages and 128-row
+key tiles, query tiles cut by the sequence end; a 4B-shaped
 sequence pair of 1000 tokens in blocks of 10 on sampled positions; and the
 workspace left reusable (a second call on it gives the same result)."""
 
@@ -70,6 +71,10 @@ CASES = [
     (1, 20, 20, 8, 8, 128),      # one block: causal self-attention only
     (1, 300, 10, 8, 2, 128),     # prefixes up to 290 rows, boundaries at every page offset
     (2, 51, 17, 8, 2, 64),
+    (1, 260, 4, 4, 2, 128),      # groups of 2: 64-position query tiles, ragged last tile
+    (1, 264, 24, 2, 2, 128),     # a tile's own rows span two key tiles (120 .. 255)
+    (2, 384, 32, 4, 4, 128),     # 128-position tiles of four blocks each
+    (1, 136, 8, 16, 8, 64),      # head_dim 64, groups of 2
 ]
 
 
