@@ -3,25 +3,31 @@
 // KV^dec at positions < s(p) = (p / b) * b and its own block's raw-embedding
 // rows at positions s(p) .. p.
 //
-// A prefill-style kernel for head_dim 128: each CTA takes 128 query rows --
+// A prefill-style kernel for head_dim 128.  A work item is 128 query rows --
 // 128 / G consecutive positions times the G query heads of one KV head, the
-// row of (position i, head j) being i * G + j -- and streams the key tiles it
-// needs once: the deep rows below the tile's last block start, then the raw-
-// embedding rows from its first block start to its last position.  Per tile,
-// S = Q K^T (tcgen05, bf16 -> f32 in TMEM), an online softmax in the log2
-// domain with the block mask, and O += P V with P split into bf16 hi + lo
-// terms (so P carries 16 significant bits).  Two S/P buffers let S(t+1) run
-// while tile t's softmax runs.
+// row of (position i, head j) being i * G + j -- and the key tiles it needs,
+// each read once: the deep rows below the item's last block start, then the
+// raw-embedding rows from its first block start to its last position.  Per
+// key tile, S = Q K^T (tcgen05, bf16 -> f32 in TMEM), an online softmax in
+// the log2 domain with the block mask, and O += P V with P split into bf16
+// hi + lo terms (P keeps 16 significant bits).  Two S/P buffers let S(t + 1)
+// run while tile t's softmax runs.
+//
+// Persistent: one CTA per SM walks the items (longest prefixes first,
+// strided over the CTAs).  Every counter runs over the CTA's whole sequence
+// of key tiles, so the next item's Q and first key tiles load, and its first
+// S runs, while the softmax warps still finish the last item's epilogue.
 //
 // Warp roles (320 threads): warps 0-7 softmax and epilogue -- warp w takes
 // TMEM lane quarter w % 4 and key / output columns [64 (w / 4), + 64), the
 // two halves of a row trading their maxima through shared memory -- warp 8
-// TMA producer, warp 9 MMA issuer and TMEM owner.
-// Every wait is bounded; a wait that gives up raises SEED_DEVERR_TIMEOUT, and
-// the CTA still drains its copies and MMAs before it frees TMEM and exits.
+// TMA producer, warp 9 MMA issuer and TMEM owner.  Every wait is bounded; a
+// wait that gives up raises SEED_DEVERR_TIMEOUT, and the CTA still drains its
+// copies and MMAs before it frees TMEM and exits.
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <atomic>
 #include <cmath>
 #include <mutex>
@@ -45,6 +51,7 @@ constexpr uint32_t kBOffV = kBOffK + 2 * kBTile;
 constexpr uint32_t kBOffCtrl = kBOffV + 2 * kBTile;
 constexpr uint32_t kBOffX = kBOffCtrl + 256;   // f32 [2 tiles][2 halves][128 rows] row maxima
 constexpr uint32_t kBOffL = kBOffX + 2048;     // f32 [2 halves][128 rows] row sums
+constexpr uint32_t kBOffE = kBOffL + 1024;     // epilogue staging: 4 KiB per softmax warp
 constexpr uint32_t kBColO = 256;               // S/P buffers [0, 256), O [256, 384)
 constexpr uint32_t kBIdescS = idesc_bf16_f32(128, kBN, 0, 0);   // K-major A and B
 constexpr uint32_t kBIdescPV = idesc_bf16_f32(128, kBD, 0, 1);  // B (V) MN-major
@@ -53,22 +60,22 @@ constexpr float kBLn2 = 0.69314718055994531f;
 constexpr unsigned kBFull = 0xffffffffu;
 
 struct BCtrl {
-  uint64_t q_full;
+  uint64_t q_full, q_empty;
   uint64_t k_full[2], k_empty[2], v_full[2], v_empty[2];
   uint64_t s_full[2], p_full[2];
   uint64_t x_full[2], l_full;                  // the softmax warps' exchanges
-  uint64_t o_full, mma_done;
+  uint64_t o_full, o_done, mma_done;
   uint32_t tmem_base;
   volatile int32_t abort_flag;
 };
-constexpr size_t kBSmem = kBOffL + 1024 + 1024;
+constexpr size_t kBSmem = kBOffE + kBSoftWarps * 4096 + 1024;
 static_assert(sizeof(BCtrl) <= 256, "control block");
 
 struct BlockTcParams {
   float* out;          // f32 [B, n, hq, D]
   float* lse;          // f32 [B, n, hq] or null
   int32_t* err;
-  int32_t B, n, blk, hq, hkv, G, P, nqt;
+  int32_t B, n, blk, hq, hkv, G, P, nqt, nitems;
   float c2;            // softmax scale * log2(e)
 };
 
@@ -111,16 +118,25 @@ __device__ __forceinline__ uint32_t key_bits(int k0, int lo, int hi) {
   return (w == 32u ? 0xffffffffu : ((1u << w) - 1u)) << a;
 }
 
-// The CTA's query tile and its key tiles.
+// Two probabilities as bf16 hi + lo pairs: hi keeps the top 16 bits of each
+// f32 (so hi + the exact f32 remainder is the value), lo the remainder
+// rounded to bf16.  First argument in the low half of each word.
+__device__ __forceinline__ void split_pair(float p0, float p1, uint32_t& hi, uint32_t& lo) {
+  const uint32_t b0 = __float_as_uint(p0), b1 = __float_as_uint(p1);
+  hi = __byte_perm(b0, b1, 0x7632);
+  lo = pack_bf16x2(p0 - __uint_as_float(b0 & 0xffff0000u), p1 - __uint_as_float(b1 & 0xffff0000u));
+}
+
+// A work item's query tile and its key tiles.
 struct BTiles {
   int b, g, p0, plast, s_lo, nd, nt;
 };
 
-__device__ __forceinline__ BTiles tiles_of(const BlockTcParams& p) {
+__device__ __forceinline__ BTiles tiles_of(const BlockTcParams& p, int item) {
   BTiles t;
   const int per = p.B * p.hkv;
-  const int qt = p.nqt - 1 - (int)(blockIdx.x / per);   // longest prefixes first
-  const int rest = (int)(blockIdx.x % per);
+  const int qt = p.nqt - 1 - item / per;       // longest prefixes first
+  const int rest = item - (item / per) * per;
   t.b = rest / p.hkv;
   t.g = rest - t.b * p.hkv;
   t.p0 = qt * p.P;
@@ -130,6 +146,19 @@ __device__ __forceinline__ BTiles tiles_of(const BlockTcParams& p) {
   t.nd = (s_hi + kBN - 1) / kBN;                          // deep tiles: rows [0, s_hi)
   t.nt = t.nd + (t.plast + 1 - t.s_lo + kBN - 1) / kBN;   // then rows [s_lo, plast]
   return t;
+}
+
+// The MMA issuer's position in the CTA's sequence of items and key tiles.
+struct BCursor {
+  int item, wi, t, nt;
+};
+
+__device__ __forceinline__ void cursor_next(BCursor& c, const BlockTcParams& p) {
+  if (++c.t < c.nt) return;
+  c.t = 0;
+  ++c.wi;
+  c.item += (int)gridDim.x;
+  c.nt = c.item < p.nitems ? tiles_of(p, c.item).nt : 0;
 }
 
 __global__ void __launch_bounds__(kBThreads, 1) block_tc_kernel(
@@ -144,6 +173,7 @@ __global__ void __launch_bounds__(kBThreads, 1) block_tc_kernel(
   if (tid == 0) pdl_trigger();
   if (tid == 0) {
     mbar_init(&ctrl->q_full, 1);
+    mbar_init(&ctrl->q_empty, 1);
     for (int i = 0; i < 2; ++i) {
       mbar_init(&ctrl->k_full[i], 1);
       mbar_init(&ctrl->k_empty[i], 1);
@@ -155,6 +185,7 @@ __global__ void __launch_bounds__(kBThreads, 1) block_tc_kernel(
     }
     mbar_init(&ctrl->l_full, kBSoftWarps);
     mbar_init(&ctrl->o_full, 1);
+    mbar_init(&ctrl->o_done, 1);
     mbar_init(&ctrl->mma_done, 1);
     ctrl->abort_flag = 0;
     fence_mbar_init();
@@ -168,7 +199,6 @@ __global__ void __launch_bounds__(kBThreads, 1) block_tc_kernel(
   tc_fence_after();
   const uint32_t tmem = ctrl->tmem_base;
   pdl_wait();
-  const BTiles T = tiles_of(p);
 
   if (warp == kBWarpProd) {
     // ---------------------------------------------------------- TMA producer
@@ -178,33 +208,40 @@ __global__ void __launch_bounds__(kBThreads, 1) block_tc_kernel(
       tma_prefetch_desc(&tm_vd);
       tma_prefetch_desc(&tm_ks);
       tma_prefetch_desc(&tm_vs);
-      mbar_arrive_expect_tx(&ctrl->q_full, kBTile);
-      tma_load_4d(smem, &tm_q, 0, T.g * p.G, T.p0, T.b, &ctrl->q_full);
-      tma_load_4d(smem + kBHalf, &tm_q, 64, T.g * p.G, T.p0, T.b, &ctrl->q_full);
-      int kiss = 0, viss = 0;                  // K and V tiles issued
-      for (int t = 0; t < T.nt; ++t) {
-        const int s = t & 1;
-        const uint32_t ph = (uint32_t)(((t >> 1) - 1) & 1);
-        const bool deep = t < T.nd;
-        const int k0 = deep ? t * kBN : T.s_lo + (t - T.nd) * kBN;
-        const CUtensorMap* mk = deep ? &tm_kd : &tm_ks;
-        const CUtensorMap* mv = deep ? &tm_vd : &tm_vs;
-        if (t >= 2 && !bpoll(&ctrl->k_empty[s], ph, ctrl, p.err)) break;
-        uint8_t* kb = smem + kBOffK + s * kBTile;
-        mbar_arrive_expect_tx(&ctrl->k_full[s], kBTile);
-        tma_load_4d(kb, mk, 0, T.g, k0, T.b, &ctrl->k_full[s]);
-        tma_load_4d(kb + kBHalf, mk, 64, T.g, k0, T.b, &ctrl->k_full[s]);
-        ++kiss;
-        if (t >= 2 && !bpoll(&ctrl->v_empty[s], ph, ctrl, p.err)) break;
-        uint8_t* vb = smem + kBOffV + s * kBTile;
-        mbar_arrive_expect_tx(&ctrl->v_full[s], kBTile);
-        tma_load_4d(vb, mv, 0, T.g, k0, T.b, &ctrl->v_full[s]);
-        tma_load_4d(vb + kBHalf, mv, 64, T.g, k0, T.b, &ctrl->v_full[s]);
-        ++viss;
+      int it = 0, qiss = 0, kiss = 0, viss = 0;   // key tiles; Q, K and V tiles issued
+      bool run = true;
+      for (int item = blockIdx.x, wi = 0; run && item < p.nitems; item += gridDim.x, ++wi) {
+        const BTiles T = tiles_of(p, item);
+        // the single Q buffer is free once every S of the previous item is done
+        if (wi > 0 && !bpoll(&ctrl->q_empty, (uint32_t)((wi - 1) & 1), ctrl, p.err)) break;
+        mbar_arrive_expect_tx(&ctrl->q_full, kBTile);
+        tma_load_4d(smem, &tm_q, 0, T.g * p.G, T.p0, T.b, &ctrl->q_full);
+        tma_load_4d(smem + kBHalf, &tm_q, 64, T.g * p.G, T.p0, T.b, &ctrl->q_full);
+        ++qiss;
+        for (int t = 0; t < T.nt; ++t, ++it) {
+          const int s = it & 1;
+          const uint32_t ph = (uint32_t)(((it >> 1) - 1) & 1);
+          const bool deep = t < T.nd;
+          const int k0 = deep ? t * kBN : T.s_lo + (t - T.nd) * kBN;
+          const CUtensorMap* mk = deep ? &tm_kd : &tm_ks;
+          const CUtensorMap* mv = deep ? &tm_vd : &tm_vs;
+          if (it >= 2 && !bpoll(&ctrl->k_empty[s], ph, ctrl, p.err)) { run = false; break; }
+          uint8_t* kb = smem + kBOffK + s * kBTile;
+          mbar_arrive_expect_tx(&ctrl->k_full[s], kBTile);
+          tma_load_4d(kb, mk, 0, T.g, k0, T.b, &ctrl->k_full[s]);
+          tma_load_4d(kb + kBHalf, mk, 64, T.g, k0, T.b, &ctrl->k_full[s]);
+          ++kiss;
+          if (it >= 2 && !bpoll(&ctrl->v_empty[s], ph, ctrl, p.err)) { run = false; break; }
+          uint8_t* vb = smem + kBOffV + s * kBTile;
+          mbar_arrive_expect_tx(&ctrl->v_full[s], kBTile);
+          tma_load_4d(vb, mv, 0, T.g, k0, T.b, &ctrl->v_full[s]);
+          tma_load_4d(vb + kBHalf, mv, 64, T.g, k0, T.b, &ctrl->v_full[s]);
+          ++viss;
+        }
       }
       // every copy this CTA started has landed before it moves on (the last
-      // fill of each ring slot; earlier fills were consumed before reuse)
-      bdrain(&ctrl->q_full, 0, p.err);
+      // fill of each buffer; earlier fills were consumed before reuse)
+      if (qiss > 0) bdrain(&ctrl->q_full, (uint32_t)((qiss - 1) & 1), p.err);
       for (int j = max(0, kiss - 2); j < kiss; ++j)
         bdrain(&ctrl->k_full[j & 1], (uint32_t)((j >> 1) & 1), p.err);
       for (int j = max(0, viss - 2); j < viss; ++j)
@@ -214,12 +251,14 @@ __global__ void __launch_bounds__(kBThreads, 1) block_tc_kernel(
   } else if (warp == kBWarpMma) {
     // ---------------------------------------------------------- MMA issuer
     if (lane == 0) {
-      int ts = 0, tp = 0;
-      bool ok = bpoll(&ctrl->q_full, 0, ctrl, p.err);
+      BCursor cs{(int)blockIdx.x, 0, 0, 0}, cp{(int)blockIdx.x, 0, 0, 0};
+      cs.nt = cp.nt = cs.item < p.nitems ? tiles_of(p, cs.item).nt : 0;
+      int ts = 0, tp = 0;                      // S and PV issued, over all items
       uint32_t idle = 0;
-      while (ok && tp < T.nt && !ctrl->abort_flag) {
+      while (cp.item < p.nitems && !ctrl->abort_flag) {
         bool did = false;
-        if (ts < T.nt && ts <= tp + 1 &&
+        if (cs.item < p.nitems && ts <= tp + 1 &&
+            (cs.t > 0 || mbar_test(&ctrl->q_full, (uint32_t)(cs.wi & 1))) &&
             mbar_test(&ctrl->k_full[ts & 1], (uint32_t)((ts >> 1) & 1))) {
           tc_fence_after();
           const uint32_t d = tmem + (uint32_t)(ts & 1) * kBN;
@@ -233,7 +272,9 @@ __global__ void __launch_bounds__(kBThreads, 1) block_tc_kernel(
           }
           mma_commit(&ctrl->s_full[ts & 1]);
           mma_commit(&ctrl->k_empty[ts & 1]);
+          if (cs.t == cs.nt - 1) mma_commit(&ctrl->q_empty);   // the item's last S
           ++ts;
+          cursor_next(cs, p);
           did = true;
         }
         if (tp < ts && mbar_test(&ctrl->p_full[tp & 1], (uint32_t)((tp >> 1) & 1)) &&
@@ -248,12 +289,14 @@ __global__ void __launch_bounds__(kBThreads, 1) block_tc_kernel(
           for (int kk = 0; kk < kBN / 16; ++kk) {
             const uint64_t bd = smem_desc_sw128(vb + kk * 2048u, kBHalf, 1024);
             const uint32_t a = pcol + 32 * (kk >> 1) + 8 * (kk & 1);
-            mma_ts(ocol, a, bd, kBIdescPV, (tp > 0 || kk > 0) ? 1u : 0u);
+            mma_ts(ocol, a, bd, kBIdescPV, (cp.t > 0 || kk > 0) ? 1u : 0u);
             mma_ts(ocol, a + 16, bd, kBIdescPV, 1u);
           }
           mma_commit(&ctrl->o_full);
           mma_commit(&ctrl->v_empty[tp & 1]);
+          if (cp.t == cp.nt - 1) mma_commit(&ctrl->o_done);    // the item's O is final
           ++tp;
+          cursor_next(cp, p);
           did = true;
         }
         if (did) {
@@ -274,136 +317,149 @@ __global__ void __launch_bounds__(kBThreads, 1) block_tc_kernel(
     const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
     float* xs = reinterpret_cast<float*>(smem + kBOffX);
     float* ls_sh = reinterpret_cast<float*>(smem + kBOffL);
-    const int pos = T.p0 + row / p.G;
-    const bool real = pos <= T.plast;
-    const int sp = (pos / p.blk) * p.blk;     // this row's block start
-    float m_used = -INFINITY, l = 0.f;
+    uint8_t* stage = smem + kBOffE + warp * 4096;
     bool ok = true;
-    for (int t = 0; t < T.nt && ok; ++t) {
-      ok = bwarp_wait(&ctrl->s_full[t & 1], (uint32_t)((t >> 1) & 1), ctrl, p.err);
-      if (!ok) break;
-      tc_fence_after();
-      const bool deep = t < T.nd;
-      const int k0 = (deep ? t * kBN : T.s_lo + (t - T.nd) * kBN) + 64 * hf;
-      const int lo = real ? (deep ? 0 : sp) : 1;
-      const int hi = real ? (deep ? sp - 1 : pos) : 0;   // visible keys [lo, hi]
-      const uint32_t scol = tmem + lane_off + (uint32_t)(t & 1) * kBN + 64u * hf;
-      uint32_t ra[32], rb[32];
-      tmem_ld32(scol, ra);
-      tmem_ld32(scol + 32, rb);
-      tmem_wait_ld();
-      const uint32_t ba = key_bits(k0, lo, hi), bb = key_bits(k0 + 32, lo, hi);
-      float mx = -INFINITY;
-#pragma unroll
-      for (int i = 0; i < 32; ++i) {
-        if ((ba >> i) & 1u) mx = fmaxf(mx, __uint_as_float(ra[i]));
-        if ((bb >> i) & 1u) mx = fmaxf(mx, __uint_as_float(rb[i]));
-      }
-      // the row's maximum over both column halves
-      float* xt = xs + (t & 1) * 256;
-      xt[hf * 128 + row] = mx;
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&ctrl->x_full[t & 1]);
-      ok = bwarp_wait(&ctrl->x_full[t & 1], (uint32_t)((t >> 1) & 1), ctrl, p.err);
-      if (!ok) break;
-      mx = fmaxf(mx, xt[(hf ^ 1) * 128 + row]);
-      const float mt = mx * p.c2;
-      bool resc = false;
-      float fo = 1.f;
-      if (mt > m_used + kBRescale) {
-        const float f = (m_used == -INFINITY) ? 0.f : ex2_approx(m_used - mt);
-        if (t > 0 && m_used != -INFINITY) {
-          resc = true;
-          fo = f;
-        }
-        l *= f;
-        m_used = mt;
-      }
-      const float mc = (m_used == -INFINITY) ? 0.f : m_used;
-      // P = 2^(s c2 - m) as bf16 hi + lo pairs, in place of S
-      float lsum = 0.f;
-      uint32_t wh[16], wl[16];
-#pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        const float p0 = ((ba >> (2 * i)) & 1u)
-                             ? ex2_approx(fmaf(__uint_as_float(ra[2 * i]), p.c2, -mc)) : 0.f;
-        const float p1 = ((ba >> (2 * i + 1)) & 1u)
-                             ? ex2_approx(fmaf(__uint_as_float(ra[2 * i + 1]), p.c2, -mc)) : 0.f;
-        lsum += p0 + p1;
-        const uint32_t hh = pack_bf16x2(p0, p1);
-        wh[i] = hh;
-        wl[i] = pack_bf16x2(p0 - bf16lo(hh), p1 - bf16hi(hh));
-      }
-      tmem_st16(scol, wh);
-      tmem_st16(scol + 16, wl);
-#pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        const float p0 = ((bb >> (2 * i)) & 1u)
-                             ? ex2_approx(fmaf(__uint_as_float(rb[2 * i]), p.c2, -mc)) : 0.f;
-        const float p1 = ((bb >> (2 * i + 1)) & 1u)
-                             ? ex2_approx(fmaf(__uint_as_float(rb[2 * i + 1]), p.c2, -mc)) : 0.f;
-        lsum += p0 + p1;
-        const uint32_t hh = pack_bf16x2(p0, p1);
-        wh[i] = hh;
-        wl[i] = pack_bf16x2(p0 - bf16lo(hh), p1 - bf16hi(hh));
-      }
-      tmem_st16(scol + 32, wh);
-      tmem_st16(scol + 48, wl);
-      tmem_wait_st();
-      l += lsum;
-      // O must be rescaled before PV(t) adds to it: wait for PV(t - 1)
-      if (__any_sync(kBFull, resc)) {
-        ok = bwarp_wait(&ctrl->o_full, (uint32_t)((t - 1) & 1), ctrl, p.err);
+    int it = 0;                               // key tiles, over all items
+    for (int item = blockIdx.x, wi = 0; ok && item < p.nitems; item += gridDim.x, ++wi) {
+      const BTiles T = tiles_of(p, item);
+      const int pos = T.p0 + row / p.G;
+      const bool real = pos <= T.plast;
+      const int sp = (pos / p.blk) * p.blk;   // this row's block start
+      float m_used = -INFINITY, l = 0.f;
+      for (int t = 0; t < T.nt; ++t, ++it) {
+        ok = bwarp_wait(&ctrl->s_full[it & 1], (uint32_t)((it >> 1) & 1), ctrl, p.err);
         if (!ok) break;
         tc_fence_after();
-        const uint32_t ocol = tmem + lane_off + kBColO + 64u * hf;
-#pragma unroll 1
-        for (int c = 0; c < 2; ++c) {
-          uint32_t r[32];
-          tmem_ld32(ocol + c * 32, r);
-          tmem_wait_ld();
+        const bool deep = t < T.nd;
+        const int k0 = (deep ? t * kBN : T.s_lo + (t - T.nd) * kBN) + 64 * hf;
+        const int lo = real ? (deep ? 0 : sp) : 1;
+        const int hi = real ? (deep ? sp - 1 : pos) : 0;   // visible keys [lo, hi]
+        const uint32_t scol = tmem + lane_off + (uint32_t)(it & 1) * kBN + 64u * hf;
+        uint32_t ra[32], rb[32];
+        tmem_ld32(scol, ra);
+        tmem_ld32(scol + 32, rb);
+        tmem_wait_ld();
+        const uint32_t ba = key_bits(k0, lo, hi), bb = key_bits(k0 + 32, lo, hi);
+        float mx = -INFINITY;
 #pragma unroll
-          for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * fo);
-          tmem_st32(ocol + c * 32, r);
+        for (int i = 0; i < 32; ++i) {
+          if ((ba >> i) & 1u) mx = fmaxf(mx, __uint_as_float(ra[i]));
+          if ((bb >> i) & 1u) mx = fmaxf(mx, __uint_as_float(rb[i]));
         }
+        // the row's maximum over both column halves
+        float* xt = xs + (it & 1) * 256;
+        xt[hf * 128 + row] = mx;
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&ctrl->x_full[it & 1]);
+        ok = bwarp_wait(&ctrl->x_full[it & 1], (uint32_t)((it >> 1) & 1), ctrl, p.err);
+        if (!ok) break;
+        mx = fmaxf(mx, xt[(hf ^ 1) * 128 + row]);
+        const float mt = mx * p.c2;
+        bool resc = false;
+        float fo = 1.f;
+        if (mt > m_used + kBRescale) {
+          const float f = (m_used == -INFINITY) ? 0.f : ex2_approx(m_used - mt);
+          if (t > 0 && m_used != -INFINITY) {
+            resc = true;
+            fo = f;
+          }
+          l *= f;
+          m_used = mt;
+        }
+        const float mc = (m_used == -INFINITY) ? 0.f : m_used;
+        // P = 2^(s c2 - m) as bf16 hi + lo pairs, in place of S
+        float lsum = 0.f;
+        uint32_t wh[16], wl[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const float p0 = ((ba >> (2 * i)) & 1u)
+                               ? ex2_approx(fmaf(__uint_as_float(ra[2 * i]), p.c2, -mc)) : 0.f;
+          const float p1 = ((ba >> (2 * i + 1)) & 1u)
+                               ? ex2_approx(fmaf(__uint_as_float(ra[2 * i + 1]), p.c2, -mc)) : 0.f;
+          lsum += p0 + p1;
+          split_pair(p0, p1, wh[i], wl[i]);
+        }
+        tmem_st16(scol, wh);
+        tmem_st16(scol + 16, wl);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const float p0 = ((bb >> (2 * i)) & 1u)
+                               ? ex2_approx(fmaf(__uint_as_float(rb[2 * i]), p.c2, -mc)) : 0.f;
+          const float p1 = ((bb >> (2 * i + 1)) & 1u)
+                               ? ex2_approx(fmaf(__uint_as_float(rb[2 * i + 1]), p.c2, -mc)) : 0.f;
+          lsum += p0 + p1;
+          split_pair(p0, p1, wh[i], wl[i]);
+        }
+        tmem_st16(scol + 32, wh);
+        tmem_st16(scol + 48, wl);
         tmem_wait_st();
+        l += lsum;
+        // O must be rescaled before PV(t) adds to it: wait for PV(t - 1)
+        if (__any_sync(kBFull, resc)) {
+          ok = bwarp_wait(&ctrl->o_full, (uint32_t)((it - 1) & 1), ctrl, p.err);
+          if (!ok) break;
+          tc_fence_after();
+          const uint32_t ocol = tmem + lane_off + kBColO + 64u * hf;
+#pragma unroll 1
+          for (int c = 0; c < 2; ++c) {
+            uint32_t r[32];
+            tmem_ld32(ocol + c * 32, r);
+            tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * fo);
+            tmem_st32(ocol + c * 32, r);
+          }
+          tmem_wait_st();
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&ctrl->p_full[it & 1]);
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&ctrl->p_full[t & 1]);
-    }
-    // epilogue: O / l once every MMA of the CTA has completed
-    if (ok) {
+      if (!ok) break;
+      // epilogue: the row sum over both halves, then O / l once the item's
+      // last PV has completed
       ls_sh[hf * 128 + row] = l;
       __syncwarp();
       if (lane == 0) mbar_arrive(&ctrl->l_full);
-      ok = bwarp_wait(&ctrl->l_full, 0, ctrl, p.err);
-    }
-    if (ok) {
+      ok = bwarp_wait(&ctrl->l_full, (uint32_t)(wi & 1), ctrl, p.err);
+      if (!ok) break;
       l += ls_sh[(hf ^ 1) * 128 + row];
-      ok = bwarp_wait(&ctrl->mma_done, 0, ctrl, p.err);
-    }
-    if (ok) {
+      ok = bwarp_wait(&ctrl->o_done, (uint32_t)(wi & 1), ctrl, p.err);
+      if (!ok) break;
       tc_fence_after();
       const uint32_t ocol = tmem + lane_off + kBColO + 64u * hf;
       const float inv = l > 0.f ? 1.f / l : 0.f;
-      const int h = T.g * p.G + row % p.G;
-      const size_t orow = ((size_t)T.b * p.n + (real ? pos : 0)) * p.hq + h;
+      // through a per-warp staging tile, so that the stores go out as whole
+      // 128-byte row pieces: lane i writes its row's 32 values, then each
+      // group of 8 lanes writes one row piece (16-byte chunks swizzled by row)
 #pragma unroll 1
-      for (int c = 0; c < 4; ++c) {
-        uint32_t r[16];
-        tmem_ld16(ocol + c * 16, r);
+      for (int c = 0; c < 2; ++c) {
+        uint32_t r[32];
+        tmem_ld32(ocol + c * 32, r);
         tmem_wait_ld();
-        if (real) {
-          float4* dp = reinterpret_cast<float4*>(p.out + orow * kBD + 64 * hf + c * 16);
 #pragma unroll
-          for (int i = 0; i < 4; ++i)
-            dp[i] = make_float4(__uint_as_float(r[4 * i]) * inv, __uint_as_float(r[4 * i + 1]) * inv,
-                                __uint_as_float(r[4 * i + 2]) * inv,
-                                __uint_as_float(r[4 * i + 3]) * inv);
+        for (int j = 0; j < 8; ++j)
+          *reinterpret_cast<float4*>(stage + lane * 128 + ((j ^ (lane & 7)) << 4)) =
+              make_float4(__uint_as_float(r[4 * j]) * inv, __uint_as_float(r[4 * j + 1]) * inv,
+                          __uint_as_float(r[4 * j + 2]) * inv, __uint_as_float(r[4 * j + 3]) * inv);
+        __syncwarp();
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const int rr = i * 4 + (lane >> 3), ch = lane & 7;
+          const int R = q4 * 32 + rr;
+          const int pr = T.p0 + R / p.G;
+          const float4 v = *reinterpret_cast<const float4*>(stage + rr * 128 + ((ch ^ (rr & 7)) << 4));
+          if (pr <= T.plast) {
+            const size_t orow = ((size_t)T.b * p.n + pr) * p.hq + T.g * p.G + R % p.G;
+            *reinterpret_cast<float4*>(p.out + orow * kBD + 64 * hf + 32 * c + 4 * ch) = v;
+          }
         }
+        __syncwarp();
       }
-      if (real && hf == 0 && p.lse != nullptr) p.lse[orow] = (m_used + log2f(l)) * kBLn2;
+      if (real && hf == 0 && p.lse != nullptr)
+        p.lse[((size_t)T.b * p.n + pos) * p.hq + T.g * p.G + row % p.G] =
+            (m_used + log2f(l)) * kBLn2;
+      tc_fence_before();
     }
   }
 
@@ -474,6 +530,9 @@ cudaError_t launch_block_tc(int32_t B, int32_t n, int32_t blk, int32_t hq, int32
   p.G = hq / hkv;
   p.P = 128 / p.G;
   p.nqt = (n + p.P - 1) / p.P;
+  const long long items = (long long)B * hkv * p.nqt;
+  if (items <= 0 || items > 0x7fffffffLL) return cudaErrorInvalidValue;
+  p.nitems = (int32_t)items;
   p.c2 = scale * 1.4426950408889634f;
   CUtensorMap tq, tkd, tvd, tks, tvs;
   if (!encode_bthd(&tq, q, B, n, hq, p.G, p.P) || !encode_bthd(&tkd, k_dec, B, n, hkv, 1, kBN) ||
@@ -491,8 +550,7 @@ cudaError_t launch_block_tc(int32_t B, int32_t n, int32_t blk, int32_t hq, int32
     if (e != cudaSuccess) return e;
     g_block_attr.fetch_or(bit, std::memory_order_acq_rel);
   }
-  const long long grid = (long long)B * hkv * p.nqt;
-  if (grid <= 0 || grid > 0x7fffffffLL) return cudaErrorInvalidValue;
+  const int grid = (int)std::min<long long>(items, std::max(1, device_sm_count()));
   return launch_pdl(block_tc_kernel, dim3((unsigned)grid), dim3(kBThreads), kBSmem, st, tq, tkd,
                     tvd, tks, tvs, p);
 }
