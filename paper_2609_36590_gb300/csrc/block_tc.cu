@@ -15,8 +15,10 @@
 //
 // Persistent: one CTA per SM walks the items (longest prefixes first,
 // strided over the CTAs).  Every counter runs over the CTA's whole sequence
-// of key tiles, so the next item's Q and first key tiles load, and its first
-// S runs, while the softmax warps still finish the last item's epilogue.
+// of key tiles, and O is double-buffered by item, so the next item's Q and
+// key tiles load and its first S and PV run while the softmax warps write
+// out the previous item: they do that epilogue after handing over the next
+// item's first P.
 //
 // Warp roles (320 threads): warps 0-7 softmax and epilogue -- warp w takes
 // TMEM lane quarter w % 4 and key / output columns [64 (w / 4), + 64), the
@@ -50,9 +52,9 @@ constexpr uint32_t kBOffK = kBTile;            // Q at 0, then the K ring, then 
 constexpr uint32_t kBOffV = kBOffK + 2 * kBTile;
 constexpr uint32_t kBOffCtrl = kBOffV + 2 * kBTile;
 constexpr uint32_t kBOffX = kBOffCtrl + 256;   // f32 [2 tiles][2 halves][128 rows] row maxima
-constexpr uint32_t kBOffL = kBOffX + 2048;     // f32 [2 halves][128 rows] row sums
-constexpr uint32_t kBOffE = kBOffL + 1024;     // epilogue staging: 4 KiB per softmax warp
-constexpr uint32_t kBColO = 256;               // S/P buffers [0, 256), O [256, 384)
+constexpr uint32_t kBOffL = kBOffX + 2048;     // f32 [2 items][2 halves][128 rows] row sums
+constexpr uint32_t kBOffE = kBOffL + 2048;     // epilogue staging: 4 KiB per softmax warp
+constexpr uint32_t kBColO = 256;               // S/P buffers [0, 256), O buffers [256, 512)
 constexpr uint32_t kBIdescS = idesc_bf16_f32(128, kBN, 0, 0);   // K-major A and B
 constexpr uint32_t kBIdescPV = idesc_bf16_f32(128, kBD, 0, 1);  // B (V) MN-major
 constexpr float kBRescale = 8.0f;
@@ -63,8 +65,8 @@ struct BCtrl {
   uint64_t q_full, q_empty;
   uint64_t k_full[2], k_empty[2], v_full[2], v_empty[2];
   uint64_t s_full[2], p_full[2];
-  uint64_t x_full[2], l_full;                  // the softmax warps' exchanges
-  uint64_t o_full, o_done, mma_done;
+  uint64_t x_full[2], l_full[2];               // the softmax warps' exchanges
+  uint64_t o_full, o_done[2], mma_done;
   uint32_t tmem_base;
   volatile int32_t abort_flag;
 };
@@ -127,6 +129,66 @@ __device__ __forceinline__ void split_pair(float p0, float p1, uint32_t& hi, uin
   lo = pack_bf16x2(p0 - __uint_as_float(b0 & 0xffff0000u), p1 - __uint_as_float(b1 & 0xffff0000u));
 }
 
+// Warp-uniform class of a 32-key chunk: 2 when every lane sees all its keys,
+// 0 when no lane sees any, 1 otherwise.
+__device__ __forceinline__ int chunk_kind(uint32_t bits) {
+  if (__all_sync(kBFull, bits == 0xffffffffu)) return 2;
+  if (__all_sync(kBFull, bits == 0u)) return 0;
+  return 1;
+}
+
+// Maximum of a chunk's visible scores (-inf if none).
+__device__ __forceinline__ float chunk_max(const uint32_t (&r)[32], uint32_t bits, int kind) {
+  if (kind == 2) {
+    float a[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) a[i] = fmaxf(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1]));
+#pragma unroll
+    for (int w = 8; w >= 1; w >>= 1)
+#pragma unroll
+      for (int i = 0; i < w; ++i) a[i] = fmaxf(a[i], a[i + w]);
+    return a[0];
+  }
+  float m = -INFINITY;
+  if (kind == 1) {
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+      m = fmaxf(m, ((bits >> i) & 1u) ? __uint_as_float(r[i]) : -INFINITY);
+  }
+  return m;
+}
+
+// P = 2^(s c2 - mc) of a chunk (0 where masked) as bf16 hi + lo pairs;
+// returns the chunk's sum of P.
+__device__ __forceinline__ float chunk_p(const uint32_t (&r)[32], uint32_t bits, int kind,
+                                         float c2, float mc, uint32_t (&wh)[16],
+                                         uint32_t (&wl)[16]) {
+  float ls = 0.f;
+  if (kind == 2) {
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const float p0 = ex2_approx(fmaf(__uint_as_float(r[2 * i]), c2, -mc));
+      const float p1 = ex2_approx(fmaf(__uint_as_float(r[2 * i + 1]), c2, -mc));
+      ls += p0 + p1;
+      split_pair(p0, p1, wh[i], wl[i]);
+    }
+  } else if (kind == 1) {
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const float x0 = ((bits >> (2 * i)) & 1u) ? fmaf(__uint_as_float(r[2 * i]), c2, -mc) : -INFINITY;
+      const float x1 =
+          ((bits >> (2 * i + 1)) & 1u) ? fmaf(__uint_as_float(r[2 * i + 1]), c2, -mc) : -INFINITY;
+      const float p0 = ex2_approx(x0), p1 = ex2_approx(x1);   // 2^-inf = +0
+      ls += p0 + p1;
+      split_pair(p0, p1, wh[i], wl[i]);
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < 16; ++i) wh[i] = wl[i] = 0u;
+  }
+  return ls;
+}
+
 // A work item's query tile and its key tiles.
 struct BTiles {
   int b, g, p0, plast, s_lo, nd, nt;
@@ -183,9 +245,11 @@ __global__ void __launch_bounds__(kBThreads, 1) block_tc_kernel(
       mbar_init(&ctrl->p_full[i], kBSoftWarps);
       mbar_init(&ctrl->x_full[i], kBSoftWarps);
     }
-    mbar_init(&ctrl->l_full, kBSoftWarps);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&ctrl->l_full[i], kBSoftWarps);
+      mbar_init(&ctrl->o_done[i], 1);
+    }
     mbar_init(&ctrl->o_full, 1);
-    mbar_init(&ctrl->o_done, 1);
     mbar_init(&ctrl->mma_done, 1);
     ctrl->abort_flag = 0;
     fence_mbar_init();
@@ -281,7 +345,7 @@ __global__ void __launch_bounds__(kBThreads, 1) block_tc_kernel(
             mbar_test(&ctrl->v_full[tp & 1], (uint32_t)((tp >> 1) & 1))) {
           tc_fence_after();
           const uint32_t pcol = tmem + (uint32_t)(tp & 1) * kBN;
-          const uint32_t ocol = tmem + kBColO;
+          const uint32_t ocol = tmem + kBColO + (uint32_t)(cp.wi & 1) * kBD;
           const uint32_t vb = sbase + kBOffV + (uint32_t)(tp & 1) * kBTile;
           // keys [16 kk, 16 kk + 16): P_hi at packed column 32 (kk / 2) + 8 (kk % 2),
           // P_lo 16 columns further
@@ -294,7 +358,7 @@ __global__ void __launch_bounds__(kBThreads, 1) block_tc_kernel(
           }
           mma_commit(&ctrl->o_full);
           mma_commit(&ctrl->v_empty[tp & 1]);
-          if (cp.t == cp.nt - 1) mma_commit(&ctrl->o_done);    // the item's O is final
+          if (cp.t == cp.nt - 1) mma_commit(&ctrl->o_done[cp.wi & 1]);   // the item's O is final
           ++tp;
           cursor_next(cp, p);
           did = true;
@@ -318,7 +382,51 @@ __global__ void __launch_bounds__(kBThreads, 1) block_tc_kernel(
     float* xs = reinterpret_cast<float*>(smem + kBOffX);
     float* ls_sh = reinterpret_cast<float*>(smem + kBOffL);
     uint8_t* stage = smem + kBOffE + warp * 4096;
-    bool ok = true;
+    // The epilogue of item wi: the row sum over both halves, then O / l
+    // through a per-warp staging tile, so that the stores go out as whole
+    // 128-byte row pieces (lane i writes its row's 32 values, then each group
+    // of 8 lanes writes one row piece; 16-byte chunks swizzled by row).
+    auto epilogue = [&](const BTiles& E, int ewi, float el, float em) -> bool {
+      if (!bwarp_wait(&ctrl->l_full[ewi & 1], (uint32_t)((ewi >> 1) & 1), ctrl, p.err)) return false;
+      el += ls_sh[(ewi & 1) * 256 + (hf ^ 1) * 128 + row];
+      if (!bwarp_wait(&ctrl->o_done[ewi & 1], (uint32_t)((ewi >> 1) & 1), ctrl, p.err)) return false;
+      tc_fence_after();
+      const uint32_t ocol = tmem + lane_off + kBColO + (uint32_t)(ewi & 1) * kBD + 64u * hf;
+      const float inv = el > 0.f ? 1.f / el : 0.f;
+#pragma unroll 1
+      for (int c = 0; c < 2; ++c) {
+        uint32_t r[32];
+        tmem_ld32(ocol + c * 32, r);
+        tmem_wait_ld();
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+          *reinterpret_cast<float4*>(stage + lane * 128 + ((j ^ (lane & 7)) << 4)) =
+              make_float4(__uint_as_float(r[4 * j]) * inv, __uint_as_float(r[4 * j + 1]) * inv,
+                          __uint_as_float(r[4 * j + 2]) * inv, __uint_as_float(r[4 * j + 3]) * inv);
+        __syncwarp();
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const int rr = i * 4 + (lane >> 3), ch = lane & 7;
+          const int R = q4 * 32 + rr;
+          const int pr = E.p0 + R / p.G;
+          const float4 v = *reinterpret_cast<const float4*>(stage + rr * 128 + ((ch ^ (rr & 7)) << 4));
+          if (pr <= E.plast) {
+            const size_t orow = ((size_t)E.b * p.n + pr) * p.hq + E.g * p.G + R % p.G;
+            *reinterpret_cast<float4*>(p.out + orow * kBD + 64 * hf + 32 * c + 4 * ch) = v;
+          }
+        }
+        __syncwarp();
+      }
+      const int epos = E.p0 + row / p.G;
+      if (epos <= E.plast && hf == 0 && p.lse != nullptr)
+        p.lse[((size_t)E.b * p.n + epos) * p.hq + E.g * p.G + row % p.G] = (em + log2f(el)) * kBLn2;
+      tc_fence_before();
+      return true;
+    };
+    bool ok = true, pend = false;             // pend: the previous item awaits its epilogue
+    BTiles PT{};
+    int pwi = 0;
+    float pl = 0.f, pm = 0.f;
     int it = 0;                               // key tiles, over all items
     for (int item = blockIdx.x, wi = 0; ok && item < p.nitems; item += gridDim.x, ++wi) {
       const BTiles T = tiles_of(p, item);
@@ -338,14 +446,10 @@ __global__ void __launch_bounds__(kBThreads, 1) block_tc_kernel(
         uint32_t ra[32], rb[32];
         tmem_ld32(scol, ra);
         tmem_ld32(scol + 32, rb);
-        tmem_wait_ld();
         const uint32_t ba = key_bits(k0, lo, hi), bb = key_bits(k0 + 32, lo, hi);
-        float mx = -INFINITY;
-#pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          if ((ba >> i) & 1u) mx = fmaxf(mx, __uint_as_float(ra[i]));
-          if ((bb >> i) & 1u) mx = fmaxf(mx, __uint_as_float(rb[i]));
-        }
+        const int ka = chunk_kind(ba), kb = chunk_kind(bb);
+        tmem_wait_ld();
+        float mx = fmaxf(chunk_max(ra, ba, ka), chunk_max(rb, bb, kb));
         // the row's maximum over both column halves
         float* xt = xs + (it & 1) * 256;
         xt[hf * 128 + row] = mx;
@@ -368,28 +472,11 @@ __global__ void __launch_bounds__(kBThreads, 1) block_tc_kernel(
         }
         const float mc = (m_used == -INFINITY) ? 0.f : m_used;
         // P = 2^(s c2 - m) as bf16 hi + lo pairs, in place of S
-        float lsum = 0.f;
         uint32_t wh[16], wl[16];
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const float p0 = ((ba >> (2 * i)) & 1u)
-                               ? ex2_approx(fmaf(__uint_as_float(ra[2 * i]), p.c2, -mc)) : 0.f;
-          const float p1 = ((ba >> (2 * i + 1)) & 1u)
-                               ? ex2_approx(fmaf(__uint_as_float(ra[2 * i + 1]), p.c2, -mc)) : 0.f;
-          lsum += p0 + p1;
-          split_pair(p0, p1, wh[i], wl[i]);
-        }
+        float lsum = chunk_p(ra, ba, ka, p.c2, mc, wh, wl);
         tmem_st16(scol, wh);
         tmem_st16(scol + 16, wl);
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const float p0 = ((bb >> (2 * i)) & 1u)
-                               ? ex2_approx(fmaf(__uint_as_float(rb[2 * i]), p.c2, -mc)) : 0.f;
-          const float p1 = ((bb >> (2 * i + 1)) & 1u)
-                               ? ex2_approx(fmaf(__uint_as_float(rb[2 * i + 1]), p.c2, -mc)) : 0.f;
-          lsum += p0 + p1;
-          split_pair(p0, p1, wh[i], wl[i]);
-        }
+        lsum += chunk_p(rb, bb, kb, p.c2, mc, wh, wl);
         tmem_st16(scol + 32, wh);
         tmem_st16(scol + 48, wl);
         tmem_wait_st();
@@ -399,7 +486,7 @@ __global__ void __launch_bounds__(kBThreads, 1) block_tc_kernel(
           ok = bwarp_wait(&ctrl->o_full, (uint32_t)((it - 1) & 1), ctrl, p.err);
           if (!ok) break;
           tc_fence_after();
-          const uint32_t ocol = tmem + lane_off + kBColO + 64u * hf;
+          const uint32_t ocol = tmem + lane_off + kBColO + (uint32_t)(wi & 1) * kBD + 64u * hf;
 #pragma unroll 1
           for (int c = 0; c < 2; ++c) {
             uint32_t r[32];
@@ -414,53 +501,24 @@ __global__ void __launch_bounds__(kBThreads, 1) block_tc_kernel(
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&ctrl->p_full[it & 1]);
-      }
-      if (!ok) break;
-      // epilogue: the row sum over both halves, then O / l once the item's
-      // last PV has completed
-      ls_sh[hf * 128 + row] = l;
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&ctrl->l_full);
-      ok = bwarp_wait(&ctrl->l_full, (uint32_t)(wi & 1), ctrl, p.err);
-      if (!ok) break;
-      l += ls_sh[(hf ^ 1) * 128 + row];
-      ok = bwarp_wait(&ctrl->o_done, (uint32_t)(wi & 1), ctrl, p.err);
-      if (!ok) break;
-      tc_fence_after();
-      const uint32_t ocol = tmem + lane_off + kBColO + 64u * hf;
-      const float inv = l > 0.f ? 1.f / l : 0.f;
-      // through a per-warp staging tile, so that the stores go out as whole
-      // 128-byte row pieces: lane i writes its row's 32 values, then each
-      // group of 8 lanes writes one row piece (16-byte chunks swizzled by row)
-#pragma unroll 1
-      for (int c = 0; c < 2; ++c) {
-        uint32_t r[32];
-        tmem_ld32(ocol + c * 32, r);
-        tmem_wait_ld();
-#pragma unroll
-        for (int j = 0; j < 8; ++j)
-          *reinterpret_cast<float4*>(stage + lane * 128 + ((j ^ (lane & 7)) << 4)) =
-              make_float4(__uint_as_float(r[4 * j]) * inv, __uint_as_float(r[4 * j + 1]) * inv,
-                          __uint_as_float(r[4 * j + 2]) * inv, __uint_as_float(r[4 * j + 3]) * inv);
-        __syncwarp();
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          const int rr = i * 4 + (lane >> 3), ch = lane & 7;
-          const int R = q4 * 32 + rr;
-          const int pr = T.p0 + R / p.G;
-          const float4 v = *reinterpret_cast<const float4*>(stage + rr * 128 + ((ch ^ (rr & 7)) << 4));
-          if (pr <= T.plast) {
-            const size_t orow = ((size_t)T.b * p.n + pr) * p.hq + T.g * p.G + R % p.G;
-            *reinterpret_cast<float4*>(p.out + orow * kBD + 64 * hf + 32 * c + 4 * ch) = v;
-          }
+        // the previous item's O (the other buffer) goes out while PV(t) runs
+        if (pend) {
+          ok = epilogue(PT, pwi, pl, pm);
+          pend = false;
+          if (!ok) break;
         }
-        __syncwarp();
       }
-      if (real && hf == 0 && p.lse != nullptr)
-        p.lse[((size_t)T.b * p.n + pos) * p.hq + T.g * p.G + row % p.G] =
-            (m_used + log2f(l)) * kBLn2;
-      tc_fence_before();
+      if (!ok) break;
+      ls_sh[(wi & 1) * 256 + hf * 128 + row] = l;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctrl->l_full[wi & 1]);
+      pend = true;
+      PT = T;
+      pwi = wi;
+      pl = l;
+      pm = m_used;
     }
+    if (ok && pend) epilogue(PT, pwi, pl, pm);
   }
 
   tc_fence_before();

@@ -75,6 +75,8 @@ CASES = [
     (1, 264, 24, 2, 2, 128),     # a tile's own rows span two key tiles (120 .. 255)
     (2, 384, 32, 4, 4, 128),     # 128-position tiles of four blocks each
     (1, 136, 8, 16, 8, 64),      # head_dim 64, groups of 2
+    (64, 20, 20, 8, 8, 128),     # 512 one-tile items: several per CTA
+    (3, 200, 10, 32, 8, 128),    # 168 items of 1 to 3 key tiles: more items than SMs
 ]
 
 
