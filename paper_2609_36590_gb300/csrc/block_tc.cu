@@ -91,6 +91,23 @@ __device__ __noinline__ bool bwait(uint64_t* bar, uint32_t parity, BCtrl* c, int
   return false;
 }
 
+// A wait on the softmax warps' critical path: try_wait without a sleep hint
+// (the thread resumes as soon as the phase completes), bounded like bwait.
+__device__ __forceinline__ bool bwait_hot(uint64_t* bar, uint32_t parity, BCtrl* c, int32_t* err) {
+  for (uint32_t i = 0; i < (1u << 22); ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((i & 63u) == 63u && c->abort_flag) return false;
+  }
+  c->abort_flag = 1;
+  raise_err(err, SEED_DEVERR_TIMEOUT);
+  return false;
+}
+
+__device__ __forceinline__ bool bwarp_hot(uint64_t* bar, uint32_t parity, BCtrl* c,
+                                          int32_t* err) {
+  return __all_sync(kBFull, bwait_hot(bar, parity, c, err));
+}
+
 __device__ __forceinline__ bool bwarp_wait(uint64_t* bar, uint32_t parity, BCtrl* c,
                                            int32_t* err) {
   return __all_sync(kBFull, bwait(bar, parity, c, err));
@@ -120,13 +137,16 @@ __device__ __forceinline__ uint32_t key_bits(int k0, int lo, int hi) {
   return (w == 32u ? 0xffffffffu : ((1u << w) - 1u)) << a;
 }
 
-// Two probabilities as bf16 hi + lo pairs: hi keeps the top 16 bits of each
-// f32 (so hi + the exact f32 remainder is the value), lo the remainder
-// rounded to bf16.  First argument in the low half of each word.
+// Two probabilities as bf16 hi + lo pairs by truncation: hi keeps the top 16
+// bits of each f32, lo the top 16 bits of the exact f32 remainder, so hi + lo
+// is within 2^-14 of the value (relative) and never above it.  First
+// argument in the low half of each word.
 __device__ __forceinline__ void split_pair(float p0, float p1, uint32_t& hi, uint32_t& lo) {
   const uint32_t b0 = __float_as_uint(p0), b1 = __float_as_uint(p1);
   hi = __byte_perm(b0, b1, 0x7632);
-  lo = pack_bf16x2(p0 - __uint_as_float(b0 & 0xffff0000u), p1 - __uint_as_float(b1 & 0xffff0000u));
+  const float r0 = p0 - __uint_as_float(b0 & 0xffff0000u);
+  const float r1 = p1 - __uint_as_float(b1 & 0xffff0000u);
+  lo = __byte_perm(__float_as_uint(r0), __float_as_uint(r1), 0x7632);
 }
 
 // Warp-uniform class of a 32-key chunk: 2 when every lane sees all its keys,
@@ -137,17 +157,24 @@ __device__ __forceinline__ int chunk_kind(uint32_t bits) {
   return 1;
 }
 
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+
 // Maximum of a chunk's visible scores (-inf if none).
 __device__ __forceinline__ float chunk_max(const uint32_t (&r)[32], uint32_t bits, int kind) {
   if (kind == 2) {
-    float a[16];
+    float a[11];
 #pragma unroll
-    for (int i = 0; i < 16; ++i) a[i] = fmaxf(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1]));
-#pragma unroll
-    for (int w = 8; w >= 1; w >>= 1)
-#pragma unroll
-      for (int i = 0; i < w; ++i) a[i] = fmaxf(a[i], a[i + w]);
-    return a[0];
+    for (int i = 0; i < 10; ++i)
+      a[i] = fmax3(__uint_as_float(r[3 * i]), __uint_as_float(r[3 * i + 1]),
+                   __uint_as_float(r[3 * i + 2]));
+    a[10] = fmaxf(__uint_as_float(r[30]), __uint_as_float(r[31]));
+    const float b0 = fmax3(a[0], a[1], a[2]), b1 = fmax3(a[3], a[4], a[5]);
+    const float b2 = fmax3(a[6], a[7], a[8]), b3 = fmaxf(a[9], a[10]);
+    return fmaxf(fmax3(b0, b1, b2), b3);
   }
   float m = -INFINITY;
   if (kind == 1) {
@@ -435,7 +462,7 @@ __global__ void __launch_bounds__(kBThreads, 1) block_tc_kernel(
       const int sp = (pos / p.blk) * p.blk;   // this row's block start
       float m_used = -INFINITY, l = 0.f;
       for (int t = 0; t < T.nt; ++t, ++it) {
-        ok = bwarp_wait(&ctrl->s_full[it & 1], (uint32_t)((it >> 1) & 1), ctrl, p.err);
+        ok = bwarp_hot(&ctrl->s_full[it & 1], (uint32_t)((it >> 1) & 1), ctrl, p.err);
         if (!ok) break;
         tc_fence_after();
         const bool deep = t < T.nd;
@@ -455,7 +482,7 @@ __global__ void __launch_bounds__(kBThreads, 1) block_tc_kernel(
         xt[hf * 128 + row] = mx;
         __syncwarp();
         if (lane == 0) mbar_arrive(&ctrl->x_full[it & 1]);
-        ok = bwarp_wait(&ctrl->x_full[it & 1], (uint32_t)((it >> 1) & 1), ctrl, p.err);
+        ok = bwarp_hot(&ctrl->x_full[it & 1], (uint32_t)((it >> 1) & 1), ctrl, p.err);
         if (!ok) break;
         mx = fmaxf(mx, xt[(hf ^ 1) * 128 + row]);
         const float mt = mx * p.c2;
@@ -483,7 +510,7 @@ __global__ void __launch_bounds__(kBThreads, 1) block_tc_kernel(
         l += lsum;
         // O must be rescaled before PV(t) adds to it: wait for PV(t - 1)
         if (__any_sync(kBFull, resc)) {
-          ok = bwarp_wait(&ctrl->o_full, (uint32_t)((it - 1) & 1), ctrl, p.err);
+          ok = bwarp_hot(&ctrl->o_full, (uint32_t)((it - 1) & 1), ctrl, p.err);
           if (!ok) break;
           tc_fence_after();
           const uint32_t ocol = tmem + lane_off + kBColO + (uint32_t)(wi & 1) * kBD + 64u * hf;
