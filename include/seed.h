@@ -417,12 +417,17 @@ seed_status_t seed_draft_layer(const seed_cfg_t* cfg, int32_t batch,
  *   k_dec, v_dec, k_spec, v_spec   bf16 [batch, n, hkv, head_dim]
  *   out        f32 [batch, n, hq, head_dim]; lse f32 [batch, n, hq] or NULL
  *   ws         seed_block_attn_workspace_bytes(...) bytes, 256-byte aligned,
- *              ZERO-FILLED before its first use (it holds the attention's
- *              counters, which every call leaves zeroed, and a paged copy of
- *              the rows that each call rewrites)
+ *              ZERO-FILLED before its first use.  head_dim 128 with 1, 2 or
+ *              4 query heads per KV head runs one tensor-core kernel that
+ *              reads q and the four inputs directly (the size is then 256
+ *              and the workspace is not touched); other shapes run the
+ *              verify kernel on one virtual sequence per block, and the
+ *              workspace holds its counters (every call leaves them zeroed)
+ *              and a paged copy of the rows that each call rewrites.
  * Errors: SEED_ERR_SHAPE (sizes, block, head_dim, group), SEED_ERR_NULL,
  * SEED_ERR_RANGE (a tensor not 16-byte aligned), SEED_ERR_WORKSPACE.
- * Device errors: none expected (as seed_verify_attn). */
+ * Device errors: none expected; a wait inside a kernel that runs out raises
+ * SEED_DEVERR_TIMEOUT (as seed_verify_attn). */
 size_t seed_block_attn_workspace_bytes(const seed_cfg_t* cfg, int32_t batch, int32_t n,
                                        int32_t block);
 seed_status_t seed_block_attn(const seed_cfg_t* cfg, int32_t batch, int32_t n, int32_t block,
