@@ -129,6 +129,15 @@ __device__ __forceinline__ void bdrain(uint64_t* bar, uint32_t parity, int32_t* 
   raise_err(err, SEED_DEVERR_TIMEOUT);
 }
 
+// Pull a 4-d box of a tensor map into L2 (no shared memory, no completion).
+__device__ __forceinline__ void tma_prefetch_l2_4d(const CUtensorMap* map, int x, int y, int z,
+                                                   int w) {
+  asm volatile("cp.async.bulk.prefetch.tensor.4d.L2.global.tile [%0, {%1, %2, %3, %4}];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y), "r"(z), "r"(w)
+               : "memory");
+}
+
 // Bits of the 32 keys k0 .. k0 + 31 that lie in [lo, hi].
 __device__ __forceinline__ uint32_t key_bits(int k0, int lo, int hi) {
   const int a = max(lo - k0, 0), e = min(hi - k0, 31);
@@ -309,6 +318,13 @@ __global__ void __launch_bounds__(kBThreads, 1) block_tc_kernel(
         tma_load_4d(smem, &tm_q, 0, T.g * p.G, T.p0, T.b, &ctrl->q_full);
         tma_load_4d(smem + kBHalf, &tm_q, 64, T.g * p.G, T.p0, T.b, &ctrl->q_full);
         ++qiss;
+        // the next item's Q is read once from HBM: start it towards L2 now, so
+        // that its load after this item's last S does not wait on HBM latency
+        if (item + (int)gridDim.x < p.nitems) {
+          const BTiles N = tiles_of(p, item + (int)gridDim.x);
+          tma_prefetch_l2_4d(&tm_q, 0, N.g * p.G, N.p0, N.b);
+          tma_prefetch_l2_4d(&tm_q, 64, N.g * p.G, N.p0, N.b);
+        }
         for (int t = 0; t < T.nt; ++t, ++it) {
           const int s = it & 1;
           const uint32_t ph = (uint32_t)(((it >> 1) - 1) & 1);
@@ -406,62 +422,27 @@ __global__ void __launch_bounds__(kBThreads, 1) block_tc_kernel(
     const int q4 = warp & 3, hf = warp >> 2;  // lane quarter, column half
     const int row = q4 * 32 + lane;
     const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
+    const int lg = p.G >> 1;                  // log2 G for G in {1, 2, 4}
     float* xs = reinterpret_cast<float*>(smem + kBOffX);
     float* ls_sh = reinterpret_cast<float*>(smem + kBOffL);
     uint8_t* stage = smem + kBOffE + warp * 4096;
-    // The epilogue of item wi: the row sum over both halves, then O / l
-    // through a per-warp staging tile, so that the stores go out as whole
-    // 128-byte row pieces (lane i writes its row's 32 values, then each group
-    // of 8 lanes writes one row piece; 16-byte chunks swizzled by row).
-    auto epilogue = [&](const BTiles& E, int ewi, float el, float em) -> bool {
-      if (!bwarp_wait(&ctrl->l_full[ewi & 1], (uint32_t)((ewi >> 1) & 1), ctrl, p.err)) return false;
-      el += ls_sh[(ewi & 1) * 256 + (hf ^ 1) * 128 + row];
-      if (!bwarp_wait(&ctrl->o_done[ewi & 1], (uint32_t)((ewi >> 1) & 1), ctrl, p.err)) return false;
-      tc_fence_after();
-      const uint32_t ocol = tmem + lane_off + kBColO + (uint32_t)(ewi & 1) * kBD + 64u * hf;
-      const float inv = el > 0.f ? 1.f / el : 0.f;
-#pragma unroll 1
-      for (int c = 0; c < 2; ++c) {
-        uint32_t r[32];
-        tmem_ld32(ocol + c * 32, r);
-        tmem_wait_ld();
-#pragma unroll
-        for (int j = 0; j < 8; ++j)
-          *reinterpret_cast<float4*>(stage + lane * 128 + ((j ^ (lane & 7)) << 4)) =
-              make_float4(__uint_as_float(r[4 * j]) * inv, __uint_as_float(r[4 * j + 1]) * inv,
-                          __uint_as_float(r[4 * j + 2]) * inv, __uint_as_float(r[4 * j + 3]) * inv);
-        __syncwarp();
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          const int rr = i * 4 + (lane >> 3), ch = lane & 7;
-          const int R = q4 * 32 + rr;
-          const int pr = E.p0 + R / p.G;
-          const float4 v = *reinterpret_cast<const float4*>(stage + rr * 128 + ((ch ^ (rr & 7)) << 4));
-          if (pr <= E.plast) {
-            const size_t orow = ((size_t)E.b * p.n + pr) * p.hq + E.g * p.G + R % p.G;
-            *reinterpret_cast<float4*>(p.out + orow * kBD + 64 * hf + 32 * c + 4 * ch) = v;
-          }
-        }
-        __syncwarp();
-      }
-      const int epos = E.p0 + row / p.G;
-      if (epos <= E.plast && hf == 0 && p.lse != nullptr)
-        p.lse[((size_t)E.b * p.n + epos) * p.hq + E.g * p.G + row % p.G] = (em + log2f(el)) * kBLn2;
-      tc_fence_before();
-      return true;
-    };
     bool ok = true, pend = false;             // pend: the previous item awaits its epilogue
     BTiles PT{};
     int pwi = 0;
-    float pl = 0.f, pm = 0.f;
+    float pm = 0.f;
     int it = 0;                               // key tiles, over all items
-    for (int item = blockIdx.x, wi = 0; ok && item < p.nitems; item += gridDim.x, ++wi) {
-      const BTiles T = tiles_of(p, item);
-      const int pos = T.p0 + row / p.G;
-      const bool real = pos <= T.plast;
-      const int sp = (pos / p.blk) * p.blk;   // this row's block start
-      float m_used = -INFINITY, l = 0.f;
-      for (int t = 0; t < T.nt; ++t, ++it) {
+    int item = blockIdx.x, wi = 0, t = 0;
+    BTiles T = tiles_of(p, item);
+    int pos = T.p0 + (row >> lg);
+    bool real = pos <= T.plast;
+    int sp = (pos / p.blk) * p.blk;           // this row's block start
+    float m_used = -INFINITY, l = 0.f;
+    // One step per key tile, then one more after the last item: a tile's step
+    // ends by handing its P to the MMA warp; the step of an item's first tile
+    // (or the final step) then writes out the previous item.
+    while (ok) {
+      const bool active = item < p.nitems;
+      if (active) {
         ok = bwarp_hot(&ctrl->s_full[it & 1], (uint32_t)((it >> 1) & 1), ctrl, p.err);
         if (!ok) break;
         tc_fence_after();
@@ -498,16 +479,24 @@ __global__ void __launch_bounds__(kBThreads, 1) block_tc_kernel(
           m_used = mt;
         }
         const float mc = (m_used == -INFINITY) ? 0.f : m_used;
-        // P = 2^(s c2 - m) as bf16 hi + lo pairs, in place of S
-        uint32_t wh[16], wl[16];
-        float lsum = chunk_p(ra, ba, ka, p.c2, mc, wh, wl);
-        tmem_st16(scol, wh);
-        tmem_st16(scol + 16, wl);
-        lsum += chunk_p(rb, bb, kb, p.c2, mc, wh, wl);
-        tmem_st16(scol + 32, wh);
-        tmem_st16(scol + 48, wl);
+        // P = 2^(s c2 - m) as bf16 hi + lo pairs, in place of S; the second
+        // chunk goes through the same code after a register copy
+        uint32_t bits = ba;
+        int kind = ka;
+#pragma unroll 1
+        for (int c = 0; c < 2; ++c) {
+          uint32_t wh[16], wl[16];
+          l += chunk_p(ra, bits, kind, p.c2, mc, wh, wl);
+          tmem_st16(scol + 32 * c, wh);
+          tmem_st16(scol + 32 * c + 16, wl);
+          if (c == 0) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) ra[i] = rb[i];
+            bits = bb;
+            kind = kb;
+          }
+        }
         tmem_wait_st();
-        l += lsum;
         // O must be rescaled before PV(t) adds to it: wait for PV(t - 1)
         if (__any_sync(kBFull, resc)) {
           ok = bwarp_hot(&ctrl->o_full, (uint32_t)((it - 1) & 1), ctrl, p.err);
@@ -528,24 +517,82 @@ __global__ void __launch_bounds__(kBThreads, 1) block_tc_kernel(
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&ctrl->p_full[it & 1]);
-        // the previous item's O (the other buffer) goes out while PV(t) runs
-        if (pend) {
-          ok = epilogue(PT, pwi, pl, pm);
-          pend = false;
-          if (!ok) break;
+      }
+      // The previous item's O (the other buffer) goes out while PV(t) runs:
+      // the row sum over both halves, then O / l through a per-warp staging
+      // tile, so that the stores go out as whole 128-byte row pieces (lane i
+      // writes its row's 32 values, then each group of 8 lanes writes one row
+      // piece; 16-byte chunks swizzled by row).
+      if (pend && (t == 0 || !active)) {
+        pend = false;
+        ok = bwarp_wait(&ctrl->l_full[pwi & 1], (uint32_t)((pwi >> 1) & 1), ctrl, p.err);
+        if (!ok) break;
+        const float el = ls_sh[(pwi & 1) * 256 + row] + ls_sh[(pwi & 1) * 256 + 128 + row];
+        ok = bwarp_wait(&ctrl->o_done[pwi & 1], (uint32_t)((pwi >> 1) & 1), ctrl, p.err);
+        if (!ok) break;
+        tc_fence_after();
+        const uint32_t ocol = tmem + lane_off + kBColO + (uint32_t)(pwi & 1) * kBD + 64u * hf;
+        const float inv = el > 0.f ? 1.f / el : 0.f;
+        // rows q4 * 32 + 4 i + lane / 8: position p0 + (q4 * 32 + 4 i) / G + (lane / 8) / G
+        const int ebase = (PT.b * p.n + PT.p0) * p.hq + PT.g * p.G;
+        const int sub = lane >> 3, ch = lane & 7;
+        const int eoff = (sub >> lg) * (p.hq - p.G) + sub;    // the lane's part of R + (R / G)(hq - G)
+#pragma unroll 1
+        for (int c = 0; c < 2; ++c) {
+          uint32_t r[32];
+          tmem_ld32(ocol + c * 32, r);
+          tmem_wait_ld();
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            *reinterpret_cast<float4*>(stage + lane * 128 + ((j ^ (lane & 7)) << 4)) =
+                make_float4(__uint_as_float(r[4 * j]) * inv, __uint_as_float(r[4 * j + 1]) * inv,
+                            __uint_as_float(r[4 * j + 2]) * inv,
+                            __uint_as_float(r[4 * j + 3]) * inv);
+          __syncwarp();
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const int rr = i * 4 + sub;
+            const int R0 = q4 * 32 + i * 4;                   // a multiple of G
+            const float4 v =
+                *reinterpret_cast<const float4*>(stage + rr * 128 + ((ch ^ (rr & 7)) << 4));
+            if (PT.p0 + ((R0 + sub) >> lg) <= PT.plast) {
+              const size_t orow = (size_t)ebase + R0 + (R0 >> lg) * (p.hq - p.G) + eoff;
+              *reinterpret_cast<float4*>(p.out + orow * kBD + 64 * hf + 32 * c + 4 * ch) = v;
+            }
+          }
+          __syncwarp();
+        }
+        const int epos = PT.p0 + (row >> lg);
+        if (epos <= PT.plast && hf == 0 && p.lse != nullptr)
+          p.lse[((size_t)PT.b * p.n + epos) * p.hq + PT.g * p.G + (row & (p.G - 1))] =
+              (pm + log2f(el)) * kBLn2;
+        tc_fence_before();
+      }
+      if (!active) break;
+      ++it;
+      if (++t == T.nt) {
+        // the item's last tile: publish its row sum and leave its epilogue
+        // for the next step that starts an item
+        ls_sh[(wi & 1) * 256 + hf * 128 + row] = l;
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&ctrl->l_full[wi & 1]);
+        pend = true;
+        PT = T;
+        pwi = wi;
+        pm = m_used;
+        item += gridDim.x;
+        ++wi;
+        t = 0;
+        if (item < p.nitems) {
+          T = tiles_of(p, item);
+          pos = T.p0 + (row >> lg);
+          real = pos <= T.plast;
+          sp = (pos / p.blk) * p.blk;
+          m_used = -INFINITY;
+          l = 0.f;
         }
       }
-      if (!ok) break;
-      ls_sh[(wi & 1) * 256 + hf * 128 + row] = l;
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&ctrl->l_full[wi & 1]);
-      pend = true;
-      PT = T;
-      pwi = wi;
-      pl = l;
-      pm = m_used;
     }
-    if (ok && pend) epilogue(PT, pwi, pl, pm);
   }
 
   tc_fence_before();
