@@ -595,9 +595,11 @@ def run_profile_blockattn(args, wl, n=1000, block=10, batch=8):
     """--profile blockattn: the decoder's block-causal training attention
     (Sec. 3) for `batch` sequences of n tokens in blocks of 10 (the paper's
     training block size) at the workload's head shape, `--reps` calls back to
-    back.  Reports the bytes the implementation moves (each block's deep
-    prefix and own rows, q in, o and lse out, plus the paged copy it builds)
-    against the HBM peak, and the attention FLOPs."""
+    back.  Reports the attention FLOPs (4 D per query head and visible key)
+    against the bf16 peak and the bytes moved against the HBM peak: on the
+    tensor-core route (head_dim 128, groups 1, 2, 4) every input read once and
+    o and lse written once; on the virtual-sequence route each block's deep
+    prefix and own rows, q in, o and lse out, plus the paged copy it builds."""
     import torch
 
     import paper_2609_36590_gb300 as seed
