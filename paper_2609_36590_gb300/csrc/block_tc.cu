@@ -10,7 +10,7 @@
 // raw-embedding rows from its first block start to its last position.  Per
 // key tile, S = Q K^T (tcgen05, bf16 -> f32 in TMEM), an online softmax in
 // the log2 domain with the block mask, and O += P V with P split into bf16
-// hi + lo terms (P keeps 16 significant bits).  Two S/P buffers let S(t + 1)
+// hi + lo terms (within 2^-14 of P, relative).  Two S/P buffers let S(t + 1)
 // run while tile t's softmax runs.
 //
 // Persistent: one CTA per SM walks the items (longest prefixes first,
