@@ -77,6 +77,7 @@ CASES = [
     (1, 136, 8, 16, 8, 64),      # head_dim 64, groups of 2
     (64, 20, 20, 8, 8, 128),     # 512 one-tile items: several per CTA
     (3, 200, 10, 32, 8, 128),    # 168 items of 1 to 3 key tiles: more items than SMs
+    (1, 40, 10, 16, 2, 128),     # head_dim 128, groups of 8: the virtual-sequence route
 ]
 
 
