@@ -231,7 +231,7 @@ def run_seed(args, rank, world, device):
     with torch.cuda.stream(stream):
         dw.run_round(0)
     stream.synchronize()
-    assert int(dw.err.item()) == 0, "device error flag raised in warm-up"
+    assert int(dw.err.item()) == 0, f"device error flag {int(dw.err.item())} raised in warm-up"
 
     graphs, timers = {}, {}
     for r in range(1, n_rounds):
@@ -284,7 +284,7 @@ def run_seed(args, rank, world, device):
                 g.replay()
     stream.synchronize()
     clocks = sampler.stop() if sampler else None
-    assert int(dw.err.item()) == 0, "device error flag raised in timed rounds"
+    assert int(dw.err.item()) == 0, f"device error flag {int(dw.err.item())} raised in timed rounds"
     got_lens = dw.ctx_lens.cpu().numpy()
     assert (got_lens == lens[n_rounds]).all(), "accepted lengths diverged from the plan"
 
@@ -432,7 +432,7 @@ def run_profile(args):
             dw.verify_attn(ins, l)
         ev[r + 1].record()
     torch.cuda.synchronize()
-    assert int(dw.err.item()) == 0, "device error flag raised"
+    assert int(dw.err.item()) == 0, f"device error flag {int(dw.err.item())} raised"
     key = (1, dec[0]) if args.profile == "draft" else dec[0]
     nbytes = attn_call_bytes(wl, "draft" if args.profile == "draft" else "verify", key, lens, k_b)
     print(json.dumps({"profile": args.profile, "workload": wl.name,
@@ -478,7 +478,7 @@ def run_profile_head(args, wl, batch=None):
         seed.seed_draft_head_topk(h, w, 0.7, ids, probs, n_sib, stop, lse, ws, err)
         ev[r + 1].record()
     torch.cuda.synchronize()
-    assert int(err.item()) == 0, "device error flag raised"
+    assert int(err.item()) == 0, f"device error flag {int(err.item())} raised"
     nbytes = V * d * 2 + B * d * 2 + B * (10 * 8 + 12)
     us = [ev[i].elapsed_time(ev[i + 1]) * 1e3 for i in range(args.reps)]
     med = float(np.median(us))
@@ -574,7 +574,7 @@ def run_profile_draftstep(args, wl):
         graph.replay()
         ev[r + 1].record()
     torch.cuda.synchronize()
-    assert int(err.item()) == 0, "device error flag raised"
+    assert int(err.item()) == 0, f"device error flag {int(err.item())} raised"
     k_b = ins["k_b_np"]
     attn = sum(attn_call_bytes(wl, "draft", (1, l), dw.lens0, k_b) for l in wl.dec_layers)
     nbytes = drafter_bytes(wl) + attn
@@ -624,7 +624,7 @@ def run_profile_blockattn(args, wl, n=1000, block=10, batch=8):
         seed.seed_block_attn(cfg, block, q, *kv, out, lse, ws, err)
         ev[r + 1].record()
     torch.cuda.synchronize()
-    assert int(err.item()) == 0, "device error flag raised"
+    assert int(err.item()) == 0, f"device error flag {int(err.item())} raised"
     R = 2 * hkv * D * 2                               # K + V bytes of one row
     nblk = n // block
     qo = n * hq * (D * (2 + 4) + 4)

@@ -220,8 +220,9 @@ seed_status_t seed_accept_commit(int32_t batch, int32_t kmax, const int32_t* dra
  *   anc       uint32 [batch, kmax+1]: bit a of anc[b, j] = node a is an
  *             ancestor of node j
  *   others    as seed_verify_attn (same workspace size)
- * Built for head_dim 128 with (hq/hkv) * (kmax+1) <= 128; other shapes
- * return SEED_ERR_UNSUPPORTED.
+ * Built for head_dim 128 with (hq/hkv) * (kmax+1) <= 128 and for head_dim
+ * 64 with (hq/hkv) * (kmax+1) <= 48; other shapes return
+ * SEED_ERR_UNSUPPORTED.
  * Device errors: SEED_DEVERR_CTX_LEN, _NQ, _PAGE. */
 seed_status_t seed_tree_verify_attn(const seed_cfg_t* cfg, int32_t batch, const void* q,
                                     const int32_t* n_nodes, const uint32_t* anc,

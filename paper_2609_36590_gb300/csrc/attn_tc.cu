@@ -49,6 +49,7 @@
 #include <cmath>
 #include <mutex>
 
+#include "attn_sched.cuh"
 #include "common.cuh"
 #include "kernels.h"
 #include "tc.cuh"
@@ -56,9 +57,10 @@
 namespace seedk {
 namespace {
 
+using namespace sched;
+
 constexpr int kD = 128;
 constexpr int kN = 128;                      // tokens (columns) per tile
-constexpr int kPagesPerTile = kN / kPage;    // 8
 constexpr int kStagesTC = 3;
 constexpr int kThreadsTC = 384;   // warps 0-7 softmax, 8 idle, 9 V loads, 10 K loads, 11 MMA
 constexpr int kWarpLoadV = 9, kWarpProducer = 10, kWarpMma = 11;
@@ -66,7 +68,6 @@ constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kColO = 256;              // O accumulators: [256, 384) and [384, 512)
 constexpr float kRescale = 8.0f;
 constexpr float kLn2 = 0.69314718055994531f;
-constexpr unsigned kFull = 0xffffffffu;
 
 constexpr int kMetaRing = 2 * kStagesTC;      // tile descriptors in flight
 
@@ -131,143 +132,6 @@ __device__ __noinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, Ctrl*
 // abort racing with the barrier's completion cannot split the warp.
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, Ctrl* c, int32_t* err) {
   return __all_sync(0xffffffffu, wait_or_abort(bar, parity, c, err));
-}
-
-// ------------------------------------------------------------- sequences
-struct SeqT {
-  int nq, nd, ncp, cvalid, lim0, tiles, bad;
-};
-
-__device__ __forceinline__ SeqT seq_of(const AttnTcParams& p, int b) {
-  SeqT s{};
-  const int L = p.ctx_lens[b];
-  const int a = p.aux[b];
-  const long long cap = (long long)p.max_pages * kPage;
-  if (p.draft) {
-    if (a < 0 || a > p.kmax) s.bad |= SEED_DEVERR_DRAFT_LEN;
-    if (L < 0 || (long long)L > cap) s.bad |= SEED_DEVERR_CTX_LEN;
-    if (s.bad || a == 0) return s;
-    s.nq = 1;
-    s.nd = a;
-    s.cvalid = L;
-    s.lim0 = L - 1;
-    s.ncp = (L + kPage - 1) / kPage;
-    s.tiles = (s.ncp + 1 + kPagesPerTile - 1) / kPagesPerTile;
-  } else {
-    if (a < 0 || a > p.kmax + 1) s.bad |= SEED_DEVERR_NQ;
-    if (L < 0 || (long long)L + a > cap) s.bad |= SEED_DEVERR_CTX_LEN;
-    if (s.bad || a == 0) return s;
-    s.nq = a;
-    s.cvalid = L + a;
-    s.lim0 = L;
-    s.ncp = (s.cvalid + kPage - 1) / kPage;
-    s.tiles = (s.ncp + kPagesPerTile - 1) / kPagesPerTile;
-  }
-  return s;
-}
-
-// ------------------------------------------------------------- partition
-// The launch's work as a line of cost units: pair (b, g) with tiles(b) > 0
-// takes kPairCost units for its fixed cost (descriptor and Q load, first-tile
-// latency, epilogue), then one unit per tile; pairs in (b, g) order.  CTA c of
-// N owns the units [start(c), start(c+1)) with start(c) = floor(c T / N) when
-// T >= N, else min(c, T), and so the tiles whose units fall there: a
-// contiguous run of pieces, and the CTAs holding one pair are consecutive.
-constexpr int kPairCost = 2;
-__device__ __forceinline__ long long range_start(long long T, int c, int N) {
-  return T >= N ? T * c / N : min((long long)c, T);
-}
-
-// The CTA whose range holds tile x (0 <= x < T).
-__device__ __forceinline__ int cta_of(long long x, long long T, int N) {
-  return T >= N ? (int)(((x + 1) * N - 1) / T) : (int)x;
-}
-
-// Cost units of all pairs of sequence b.
-__device__ __forceinline__ long long seq_cost(const AttnTcParams& p, int tiles) {
-  return tiles > 0 ? (long long)p.hkv * (tiles + kPairCost) : 0;
-}
-
-// Warp-cooperative: T.
-__device__ __noinline__ long long total_cost(const AttnTcParams& p, int lane) {
-  long long tot = 0;
-  for (int b = lane; b < p.B; b += 32) tot += seq_cost(p, seq_of(p, b).tiles);
-  for (int o = 16; o; o >>= 1) tot += __shfl_xor_sync(kFull, tot, o);
-  return tot;
-}
-
-// A window of 32 sequences [wb, wb + 32); lane i holds sequence wb + i.
-struct SeqWin {
-  int wb;
-  SeqT mine;
-};
-
-__device__ __forceinline__ SeqT seq_or_empty(const AttnTcParams& p, int b) {
-  return b < p.B ? seq_of(p, b) : SeqT{};
-}
-
-__device__ __forceinline__ SeqT win_get(const SeqWin& w, int b) {
-  const int src = b - w.wb;
-  SeqT s;
-  s.nq = __shfl_sync(kFull, w.mine.nq, src);
-  s.nd = __shfl_sync(kFull, w.mine.nd, src);
-  s.ncp = __shfl_sync(kFull, w.mine.ncp, src);
-  s.cvalid = __shfl_sync(kFull, w.mine.cvalid, src);
-  s.lim0 = __shfl_sync(kFull, w.mine.lim0, src);
-  s.tiles = __shfl_sync(kFull, w.mine.tiles, src);
-  s.bad = 0;
-  return s;
-}
-
-// Warp-cooperative: the pair (sequence b, KV head g) whose units hold unit
-// x < T, the first unit pc of that pair, and the first tile t at or after x
-// (0 when x falls in the pair's fixed-cost units); with the window that holds b.
-__device__ __noinline__ void locate(const AttnTcParams& p, long long x, int lane, SeqWin& w,
-                                    int& b, int& g, int& t, long long& pc) {
-  long long base = 0;
-  for (w.wb = 0; w.wb < p.B; w.wb += 32) {
-    w.mine = seq_or_empty(p, w.wb + lane);
-    const long long a = seq_cost(p, w.mine.tiles);
-    long long inc = a;
-    for (int o = 1; o < 32; o <<= 1) {
-      const long long v = __shfl_up_sync(kFull, inc, o);
-      if (lane >= o) inc += v;
-    }
-    const long long tot = __shfl_sync(kFull, inc, 31);
-    if (x < base + tot) {
-      const unsigned m = __ballot_sync(kFull, base + inc - a <= x && x < base + inc);
-      const int src = __ffs(m) - 1;
-      const long long sb = base + __shfl_sync(kFull, inc - a, src);
-      const int per = __shfl_sync(kFull, w.mine.tiles, src) + kPairCost;
-      b = w.wb + src;
-      g = (int)((x - sb) / per);
-      pc = sb + (long long)g * per;
-      t = (int)max(0LL, x - pc - kPairCost);
-      return;
-    }
-    base += tot;
-  }
-  b = p.B;
-  g = t = 0;
-  pc = 0;
-}
-
-// Warp-cooperative: the next sequence after b with at least one tile (p.B if
-// none), moving the window forward as needed.
-__device__ __noinline__ void next_seq(const AttnTcParams& p, int lane, SeqWin& w, int& b) {
-  for (;;) {
-    const unsigned m = __ballot_sync(kFull, w.mine.tiles > 0 && w.wb + lane > b);
-    if (m) {
-      b = w.wb + __ffs(m) - 1;
-      return;
-    }
-    w.wb += 32;
-    if (w.wb >= p.B) {
-      b = p.B;
-      return;
-    }
-    w.mine = seq_or_empty(p, w.wb + lane);
-  }
 }
 
 // ------------------------------------------------------------- the kernel
@@ -414,6 +278,21 @@ constexpr int kMergeThreads = 256;
 constexpr int kMergeRows = kMergeThreads / 32;
 constexpr int kMergeBatch = 8;
 
+// Per-lane slice of a record row: D / 32 consecutive floats (4 for D = 128,
+// 2 for D = 64) moved as one vector.
+template <int D> struct MergeVec;
+template <> struct MergeVec<128> {
+  using T = float4;
+  __device__ static void to(const T& v, float* f) { f[0] = v.x; f[1] = v.y; f[2] = v.z; f[3] = v.w; }
+  __device__ static T from(const float* f) { return make_float4(f[0], f[1], f[2], f[3]); }
+};
+template <> struct MergeVec<64> {
+  using T = float2;
+  __device__ static void to(const T& v, float* f) { f[0] = v.x; f[1] = v.y; }
+  __device__ static T from(const float* f) { return make_float2(f[0], f[1]); }
+};
+
+template <int D>
 __global__ void __launch_bounds__(kMergeThreads) attn_merge_kernel(const AttnTcParams p) {
   __shared__ long long sh_pc;
   __shared__ int sh_b, sh_g;
@@ -481,18 +360,22 @@ __global__ void __launch_bounds__(kMergeThreads) attn_merge_kernel(const AttnTcP
   // before the pair (then it holds the previous pair's last tile, unit pc - 1)
   const int slot_lo = 2 * c_lo + (range_start(T, c_lo, p.nctas) >= pc ? 0 : 1);
   const int Rmax = p.G * p.W1;
-  const size_t REC = (size_t)Rmax * (kD + 1);
+  const size_t REC = (size_t)Rmax * (D + 1);
+  using V = MergeVec<D>;
+  constexpr int kPer = D / 32;
   float M = -INFINITY, S = 0.f;
-  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  float acc[kPer];
+#pragma unroll
+  for (int e = 0; e < kPer; ++e) acc[e] = 0.f;
   for (int i0 = 0; i0 < nseg; i0 += kMergeBatch) {
     float li[kMergeBatch];
-    float4 x[kMergeBatch];
+    typename V::T x[kMergeBatch];
 #pragma unroll
     for (int u = 0; u < kMergeBatch; ++u) {
       const int i = min(i0 + u, nseg - 1);
       const float* rc = p.part + (size_t)(i == 0 ? slot_lo : 2 * (c_lo + i)) * REC;
-      li[u] = (i0 + u < nseg) ? __ldcg(rc + (size_t)kD * Rmax + r) : -INFINITY;
-      x[u] = __ldcg(reinterpret_cast<const float4*>(rc + (size_t)r * kD) + lane);
+      li[u] = (i0 + u < nseg) ? __ldcg(rc + (size_t)D * Rmax + r) : -INFINITY;
+      x[u] = __ldcg(reinterpret_cast<const typename V::T*>(rc + (size_t)r * D) + lane);
     }
 #pragma unroll
     for (int u = 0; u < kMergeBatch; ++u) {
@@ -501,59 +384,28 @@ __global__ void __launch_bounds__(kMergeThreads) attn_merge_kernel(const AttnTcP
       if (li[u] > M) {
         const float f = ex2_approx(M - li[u]);   // 0 for the first piece
         S *= f;
-        acc.x *= f;
-        acc.y *= f;
-        acc.z *= f;
-        acc.w *= f;
+#pragma unroll
+        for (int e = 0; e < kPer; ++e) acc[e] *= f;
         M = li[u];
       } else {
         w = ex2_approx(li[u] - M);
       }
       S += w;
-      acc.x = fmaf(w, x[u].x, acc.x);
-      acc.y = fmaf(w, x[u].y, acc.y);
-      acc.z = fmaf(w, x[u].z, acc.z);
-      acc.w = fmaf(w, x[u].w, acc.w);
+      float xv[kPer];
+      V::to(x[u], xv);
+#pragma unroll
+      for (int e = 0; e < kPer; ++e) acc[e] = fmaf(w, xv[e], acc[e]);
     }
   }
   const float inv = 1.f / S;
   const int j = r / p.G;
   const size_t orow = ((size_t)b * p.W1 + j) * p.hq + g * p.G + (r - j * p.G);
-  reinterpret_cast<float4*>(p.out + orow * kD)[lane] =
-      make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
+  float res[kPer];
+#pragma unroll
+  for (int e = 0; e < kPer; ++e) res[e] = acc[e] * inv;
+  reinterpret_cast<typename V::T*>(p.out + orow * D)[lane] = V::from(res);
   if (lane == 0 && p.lse != nullptr) p.lse[orow] = (M + log2f(S)) * kLn2;
 }
-
-// Tensor maps of the paged cache for boxes of 1, 2, 4 and 8 consecutive pages
-// (64 head dims x 16 rows x 1 KV head x n pages): n pages whose ids follow one
-// another are one copy, and land as 16 n consecutive 128-byte rows, the
-// swizzled K-major layout the MMAs read.
-struct PageMaps {
-  CUtensorMap k[4];
-  CUtensorMap v[4];
-};
-
-// Warp-cooperative: the copy box that lane s < 8 issues for page slot s of a
-// tile.  Runs of slots holding consecutive page ids are cut greedily into
-// boxes of 8, 4, 2 and 1 pages; the result is the box size if slot s starts a
-// box, else 0.  A slot at offset o of a run of n slots starts a box of
-// 2^floor(log2(n - o)) pages exactly when n with the bits below that box size
-// cleared equals o.
-__device__ __forceinline__ int box_size(int pid, int lane) {
-  const int pid_next = __shfl_down_sync(kFull, pid, 1);
-  const uint32_t valid = __ballot_sync(kFull, lane < kPagesPerTile && pid >= 0) & 0xffu;
-  const uint32_t cont =
-      __ballot_sync(kFull, lane < kPagesPerTile - 1 && pid >= 0 && pid_next == pid + 1) & 0x7fu;
-  if (lane >= kPagesPerTile || !((valid >> lane) & 1u)) return 0;
-  const uint32_t starts = valid & ~(cont << 1) & 0xffu;
-  const int r = 31 - __clz((int)(starts & ((2u << lane) - 1u)));   // first slot of the run
-  const int n = lane + __ffs((int)~(cont >> lane)) - r;            // slots in the run
-  const int o = lane - r;
-  const int sz = 1 << (31 - __clz(n - o));
-  return (n & ~(2 * sz - 1)) == o ? sz : 0;
-}
-
-__device__ __forceinline__ int log2_box(int sz) { return sz >= 8 ? 3 : sz >= 4 ? 2 : sz >= 2 ? 1 : 0; }
 
 // No __launch_bounds__: with it ptxas budgets the 320-thread block like a
 // 384-thread one and spills in the per-tile loop; without it the kernel fits
@@ -1066,9 +918,12 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
-// 4-d bf16 tensor map, innermost dimension = 128 head dims, 128-byte swizzle.
-bool encode_4d(CUtensorMap* map, const void* base, const cuuint64_t dims[4],
-               const cuuint64_t strides[3], const cuuint32_t box[4]) {
+}  // namespace
+
+// 4-d bf16 tensor map, innermost box of 64 elements (128 bytes), 128-byte
+// swizzle.
+bool encode_4d_bf16(CUtensorMap* map, const void* base, const cuuint64_t dims[4],
+                    const cuuint64_t strides[3], const cuuint32_t box[4]) {
   EncodeTiledFn fn = encode_fn();
   if (fn == nullptr) return false;
   const cuuint32_t elem[4] = {1, 1, 1, 1};
@@ -1077,9 +932,17 @@ bool encode_4d(CUtensorMap* map, const void* base, const cuuint64_t dims[4],
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+namespace {
 std::atomic<uint64_t> g_tc_attr_set{0};
-
 }  // namespace
+
+cudaError_t launch_attn_merge(const AttnTcParams& prm, int head_dim, cudaStream_t st) {
+  if (prm.nctas < 2) return cudaSuccess;        // one CTA: no pair is shared
+  const dim3 mgrid(prm.nctas - 1, (prm.G * prm.W1 + kMergeRows - 1) / kMergeRows);
+  return head_dim == 64
+             ? launch_pdl(attn_merge_kernel<64>, mgrid, dim3(kMergeThreads), 0, st, prm)
+             : launch_pdl(attn_merge_kernel<128>, mgrid, dim3(kMergeThreads), 0, st, prm);
+}
 
 bool attn_tc_supported(int head_dim, int group, int w1) {
   return head_dim == kD && group * w1 <= 128;
@@ -1098,7 +961,7 @@ cudaError_t launch_attn_tc(const AttnTcParams& prm, const void* q, const void* k
     const cuuint64_t strides[3] = {kD * 2ull, (cuuint64_t)prm.hq * kD * 2ull,
                                    W1 * prm.hq * kD * 2ull};
     const cuuint32_t box[4] = {64, (cuuint32_t)prm.G, (cuuint32_t)W1, 1};
-    if (!encode_4d(&tq, q, dims, strides, box)) return cudaErrorInvalidValue;
+    if (!encode_4d_bf16(&tq, q, dims, strides, box)) return cudaErrorInvalidValue;
   }
   {
     const cuuint64_t dims[4] = {kD, (cuuint64_t)kPage, (cuuint64_t)prm.hkv,
@@ -1107,8 +970,8 @@ cudaError_t launch_attn_tc(const AttnTcParams& prm, const void* q, const void* k
                                    (cuuint64_t)prm.hkv * kPage * kD * 2ull};
     for (int i = 0; i < 4; ++i) {
       const cuuint32_t box[4] = {64, (cuuint32_t)kPage, 1, 1u << i};
-      if (!encode_4d(&pm.k[i], k_cache, dims, strides, box)) return cudaErrorInvalidValue;
-      if (!encode_4d(&pm.v[i], v_cache, dims, strides, box)) return cudaErrorInvalidValue;
+      if (!encode_4d_bf16(&pm.k[i], k_cache, dims, strides, box)) return cudaErrorInvalidValue;
+      if (!encode_4d_bf16(&pm.v[i], v_cache, dims, strides, box)) return cudaErrorInvalidValue;
     }
   }
   if (prm.draft) {
@@ -1118,8 +981,8 @@ cudaError_t launch_attn_tc(const AttnTcParams& prm, const void* q, const void* k
     const cuuint64_t strides[3] = {kD * 2ull, (cuuint64_t)prm.kmax * kD * 2ull,
                                    (cuuint64_t)prm.hkv * prm.kmax * kD * 2ull};
     const cuuint32_t box[4] = {64, (cuuint32_t)kPage, 1, 1};
-    if (!encode_4d(&tdk, draft_k, dims, strides, box)) return cudaErrorInvalidValue;
-    if (!encode_4d(&tdv, draft_v, dims, strides, box)) return cudaErrorInvalidValue;
+    if (!encode_4d_bf16(&tdk, draft_k, dims, strides, box)) return cudaErrorInvalidValue;
+    if (!encode_4d_bf16(&tdv, draft_v, dims, strides, box)) return cudaErrorInvalidValue;
   } else {
     tdk = pm.k[0];
     tdv = pm.v[0];
@@ -1137,13 +1000,11 @@ cudaError_t launch_attn_tc(const AttnTcParams& prm, const void* q, const void* k
   e = launch_pdl(attn_tc_kernel, dim3(prm.nctas), dim3(kThreadsTC), kSmemTC, st, tq, pm, tdk, tdv,
                  prm);
   if (e != cudaSuccess) return e;
-  if (prm.nctas < 2) return cudaSuccess;        // one CTA: no pair is shared
-  const dim3 mgrid(prm.nctas - 1, (prm.G * prm.W1 + kMergeRows - 1) / kMergeRows);
-  return launch_pdl(attn_merge_kernel, mgrid, dim3(kMergeThreads), 0, st, prm);
+  return launch_attn_merge(prm, kD, st);
 }
 
-size_t attn_tc_part_bound(int32_t group, int32_t w1) {
-  return 2 * (size_t)kTcMaxCtas * group * w1 * (kD + 1) * sizeof(float);
+size_t attn_tc_part_bound(int32_t group, int32_t w1, int32_t head_dim) {
+  return 2 * (size_t)kTcMaxCtas * group * w1 * (head_dim + 1) * sizeof(float);
 }
 
 }  // namespace seedk

@@ -167,13 +167,29 @@ struct AttnTcParams {
   int32_t W1;                 // query positions per sequence: kmax+1 (verify) or 1 (draft)
   int32_t nctas;              // CTAs of the attention kernel (static tile partition)
   float scale_log2;
+  // raw inputs for the keys-as-rows kernel's exact recomputation of a piece
+  // (bf16): q [B, W1, hq, D], the paged caches, the draft scratch (draft only)
+  const uint16_t* q;
+  const uint16_t* k_cache;
+  const uint16_t* v_cache;
+  const uint16_t* draft_k;
+  const uint16_t* draft_v;
+  int32_t D;
 };
 
 bool attn_tc_supported(int head_dim, int group, int w1);
 int attn_tc_ctas();
-size_t attn_tc_part_bound(int32_t group, int32_t w1);
+// Workspace bytes of the split records of either tensor-core kernel.
+size_t attn_tc_part_bound(int32_t group, int32_t w1, int32_t head_dim);
 cudaError_t launch_attn_tc(const AttnTcParams& p, const void* q, const void* k_cache,
                            const void* v_cache, const void* draft_k, const void* draft_v,
                            cudaStream_t st);
+
+// Keys-as-rows tensor-core attention for at most 64 query rows per KV head
+// (attn_kt.cu); head_dim 64 or 128.
+bool attn_kt_supported(int head_dim, int group, int w1);
+cudaError_t launch_attn_kt(const AttnTcParams& p, int head_dim, const void* q,
+                           const void* k_cache, const void* v_cache, const void* draft_k,
+                           const void* draft_v, cudaStream_t st);
 
 }  // namespace seedk

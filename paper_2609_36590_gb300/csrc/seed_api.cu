@@ -90,8 +90,9 @@ seed_status_t run_decode(const seed_cfg_t* cfg, int32_t batch, bool verify, cons
   return finish(seedk::launch_decode(p, cfg->head_dim, G, static_cast<cudaStream_t>(stream)));
 }
 
-// Draft / verify attention on the tensor cores (head_dim 128, all query rows
-// of a KV head in one 128-row tile).
+// Draft / verify attention on the tensor cores: the keys-as-rows kernel for
+// head_dim 64 when the R = G * W1 query rows of a KV head fit 48 MMA
+// columns, the query-rows kernel for head_dim 128 (R <= 128).
 seed_status_t run_attn_tc(const seed_cfg_t* cfg, int32_t batch, bool draft, const void* q,
                           const int32_t* aux, const seed_kv_t& kv, const void* draft_k,
                           const void* draft_v, const int32_t* ctx_lens, float* out, float* lse,
@@ -102,6 +103,7 @@ seed_status_t run_attn_tc(const seed_cfg_t* cfg, int32_t batch, bool draft, cons
   const size_t cb = kSchedBytes + counters_bytes(cfg, batch);
   const int ctas = seedk::attn_tc_ctas();
   const size_t need = cb + 2 * (size_t)ctas * G * W1 * (cfg->head_dim + 1) * sizeof(float);
+  const bool kt = seedk::attn_kt_supported(cfg->head_dim, G, W1);
   if (ws_bytes < need) return SEED_ERR_WORKSPACE;
   seedk::AttnTcParams p{};
   p.page_table = kv.page_table;
@@ -123,11 +125,25 @@ seed_status_t run_attn_tc(const seed_cfg_t* cfg, int32_t batch, bool draft, cons
   p.W1 = W1;
   p.nctas = ctas;
   p.scale_log2 = scale_of(cfg) * 1.4426950408889634f;
-  return finish(seedk::launch_attn_tc(p, q, kv.k, kv.v, draft_k, draft_v,
-                                      static_cast<cudaStream_t>(stream)));
+  p.q = static_cast<const uint16_t*>(q);
+  p.k_cache = static_cast<const uint16_t*>(kv.k);
+  p.v_cache = static_cast<const uint16_t*>(kv.v);
+  p.draft_k = static_cast<const uint16_t*>(draft_k);
+  p.draft_v = static_cast<const uint16_t*>(draft_v);
+  p.D = cfg->head_dim;
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  return finish(kt ? seedk::launch_attn_kt(p, cfg->head_dim, q, kv.k, kv.v, draft_k, draft_v, st)
+                   : seedk::launch_attn_tc(p, q, kv.k, kv.v, draft_k, draft_v, st));
 }
 
 bool misaligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) != 0; }
+
+// Whether a launch with R = group * w1 query rows per KV head runs on one of
+// the tensor-core kernels.
+bool tc_path(int head_dim, int group, int w1) {
+  return seedk::attn_kt_supported(head_dim, group, w1) ||
+         seedk::attn_tc_supported(head_dim, group, w1);
+}
 
 }  // namespace
 
@@ -155,10 +171,10 @@ size_t seed_workspace_bytes(const seed_cfg_t* cfg, int32_t batch) {
   const int G = cfg->hq / cfg->hkv;
   const int32_t nv_max = batch * (cfg->kmax + 1);
   size_t part = seedk::decode_workspace_bound(nv_max, cfg->hkv, G, cfg->head_dim);
-  if (seedk::attn_tc_supported(cfg->head_dim, G, 1))
-    part = std::max(part, seedk::attn_tc_part_bound(G, 1));
-  if (seedk::attn_tc_supported(cfg->head_dim, G, cfg->kmax + 1))
-    part = std::max(part, seedk::attn_tc_part_bound(G, cfg->kmax + 1));
+  if (tc_path(cfg->head_dim, G, 1))
+    part = std::max(part, seedk::attn_tc_part_bound(G, 1, cfg->head_dim));
+  if (tc_path(cfg->head_dim, G, cfg->kmax + 1))
+    part = std::max(part, seedk::attn_tc_part_bound(G, cfg->kmax + 1, cfg->head_dim));
   return kSchedBytes + counters_bytes(cfg, batch) + round_up(part, kAlign);
 }
 
@@ -194,7 +210,7 @@ seed_status_t seed_draft_attn(const seed_cfg_t* cfg, int32_t batch, const void* 
       misaligned16(draft_k) || misaligned16(draft_v))
     return SEED_ERR_RANGE;
   if ((reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)) != 0) return SEED_ERR_WORKSPACE;
-  if (seedk::attn_tc_supported(cfg->head_dim, cfg->hq / cfg->hkv, 1))
+  if (tc_path(cfg->head_dim, cfg->hq / cfg->hkv, 1))
     return run_attn_tc(cfg, batch, true, q, draft_lens, ctx_kv, draft_k, draft_v, ctx_lens, out,
                        lse, ws, ws_bytes, err_flag, stream);
   return run_decode(cfg, batch, false, q, ctx_kv, draft_k, draft_v, ctx_lens, draft_lens, out, lse,
@@ -231,7 +247,7 @@ seed_status_t seed_verify_attn(const seed_cfg_t* cfg, int32_t batch, const void*
   if ((st = check_kv(kv)) != SEED_OK) return st;
   if (misaligned16(q) || misaligned16(kv.k) || misaligned16(kv.v)) return SEED_ERR_RANGE;
   if ((reinterpret_cast<uintptr_t>(ws) & (kAlign - 1)) != 0) return SEED_ERR_WORKSPACE;
-  if (seedk::attn_tc_supported(cfg->head_dim, cfg->hq / cfg->hkv, cfg->kmax + 1))
+  if (tc_path(cfg->head_dim, cfg->hq / cfg->hkv, cfg->kmax + 1))
     return run_attn_tc(cfg, batch, false, q, n_q, kv, nullptr, nullptr, ctx_lens, out, lse, ws,
                        ws_bytes, err_flag, stream);
   return run_decode(cfg, batch, true, q, kv, nullptr, nullptr, ctx_lens, n_q, out, lse, ws,
@@ -245,8 +261,7 @@ seed_status_t seed_tree_verify_attn(const seed_cfg_t* cfg, int32_t batch, const 
   seed_status_t st = check_cfg(cfg);
   if (st != SEED_OK) return st;
   if (batch < 0) return SEED_ERR_SHAPE;
-  if (!seedk::attn_tc_supported(cfg->head_dim, cfg->hq / cfg->hkv, cfg->kmax + 1))
-    return SEED_ERR_UNSUPPORTED;
+  if (!tc_path(cfg->head_dim, cfg->hq / cfg->hkv, cfg->kmax + 1)) return SEED_ERR_UNSUPPORTED;
   if (batch == 0) return SEED_OK;
   if (!q || !n_nodes || !anc || !ctx_lens || !out || !ws || !err_flag) return SEED_ERR_NULL;
   if ((st = check_kv(kv)) != SEED_OK) return st;

@@ -143,7 +143,9 @@ def test_tree_host_checks(lib):
     assert tv(c, anc=None) == ERR_NULL
     assert tv(c, q=None) == ERR_NULL
     assert tv(c, ws_bytes=64) == ERR_WS
-    assert tv(cfg(head_dim=64)) == ERR_UNSUP              # tensor-core path only
+    # tensor-core kernels only: head_dim 64 takes at most 64 query rows per KV
+    # head, head_dim 128 at most 128
+    assert tv(cfg(head_dim=64, hq=16, hkv=2, kmax=8)) == ERR_UNSUP   # 8 * 9 rows > 64
     assert tv(cfg(hq=64, hkv=8, kmax=16)) == ERR_UNSUP     # 8 * 17 rows > one 128-row tile
     args = [FAKE] * 5 + [8, 16] + [FAKE] * 6
     assert lib.seed_tree_accept_commit(0, 4, *args, None) == OK

@@ -141,6 +141,63 @@ def test_verify_attention_matches_oracle(S, case):
         assert_close(lse[b, :n], l, f"verify lse b={b}")
 
 
+def spike_rows(c, which, step, log2_gap):
+    """Key rows that score log2_gap (in log2 units of the softmax) above a
+    typical score for query head G g of KV head g: every step-th visible row
+    from position 130 on (past the first 128-key tile), plus, for the draft
+    call, the first draft row.  Each is a multiple of that query row."""
+    B, hkv, D = c["rows_k"].shape[0], c["rows_k"].shape[2], c["rows_k"].shape[3]
+    hq = c["q_draft"].shape[1]
+    G = hq // hkv
+    lg2e = 1.0 / np.log(2.0)
+    for b in range(B):
+        L = int(c["lens"][b])
+        for g in range(hkv):
+            q = f64(c["q_draft"][b, g * G] if which == "draft" else c["q_verify"][b, 0, g * G])
+            alpha = log2_gap / (c["scale"] * lg2e * float(q @ q))
+            row = gen.f32_to_bf16_bits((alpha * q).astype(np.float32))
+            for pos in range(130, L, step):
+                c["rows_k"][b, pos, g] = row
+            if which == "draft":
+                c["draft_k"][b, g, 0] = row
+
+
+@pytest.mark.parametrize("case", [(10, 32, 8, 128, 4, 1100, True, 1.0),
+                                  (10, 16, 8, 64, 2, 900, True, 1.0)],
+                         ids=["D128_G4", "D64_G2"])
+@pytest.mark.parametrize("gap", [40.0, 300.0], ids=["gap40", "gap300"])
+def test_late_score_spikes_match_oracle(S, case, gap):
+    """Scores far above the first tile's maximum, in later tiles and in the
+    draft rows: a gap below 64 (log2) stays on the fast path with weights up
+    to 2^gap; a gap of 300 takes the exact recomputation of the piece."""
+    c = make(S, 3, case)
+    spike_rows(c, "draft", 97, gap)
+    out, lse = run_draft(S, c, kv_for(S, c, c["lens"]))
+    assert int(c["err"].item()) == 0
+    for b in range(case[0]):
+        dl, L = int(c["draft_lens"][b]), int(c["lens"][b])
+        if dl == 0:
+            continue
+        o, l = OAT.draft_attention_seq(
+            f64(c["q_draft"][b]), f64(c["rows_k"][b, :L]), f64(c["rows_v"][b, :L]),
+            f64(c["draft_k"][b, :, :dl].transpose(1, 0, 2)),
+            f64(c["draft_v"][b, :, :dl].transpose(1, 0, 2)), c["scale"])
+        assert_close(out[b], o, f"draft o b={b} L={L} dl={dl}")
+        assert_close(lse[b], l, f"draft lse b={b}")
+    c = make(S, 4, case)
+    spike_rows(c, "verify", 113, gap)
+    out, lse = run_verify(S, c, kv_for(S, c, c["lens"] + c["n_q"]))
+    assert int(c["err"].item()) == 0
+    for b in range(case[0]):
+        n, L = int(c["n_q"][b]), int(c["lens"][b])
+        if n == 0:
+            continue
+        o, l = OAT.verify_attention_seq(f64(c["q_verify"][b, :n]), f64(c["rows_k"][b, :L + n]),
+                                        f64(c["rows_v"][b, :L + n]), L, c["scale"])
+        assert_close(out[b, :n], o, f"verify o b={b} L={L} n={n}")
+        assert_close(lse[b, :n], l, f"verify lse b={b}")
+
+
 def test_deterministic_and_page_order_invariant(S):
     case = (5, 32, 8, 128, 8, 1100, True, 1.0)
     c = make(S, 3, case)
