@@ -445,6 +445,7 @@ __global__ void __launch_bounds__(kThreadsKT, 1)
       tma_prefetch_desc(&tm_dv);
     }
   }
+  if (warp == kWarpProdK) prefetch_lens_l2(p, lane);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -481,6 +482,10 @@ __global__ void __launch_bounds__(kThreadsKT, 1)
     int b = p.B, g = 0, t0 = 0;
     long long pc = 0;
     if (x < x1) locate(p, x, lane, win, b, g, t0, pc);
+    {
+      const SeqT s0 = b < p.B ? win_get(win, b) : SeqT{};
+      if (lane == 0) write_merge_plan(p, T, x, x1, b, g, t0, pc, s0);
+    }
     int tk = 0, uo = 0;
     bool ok = true;
     int pid_a = -1, pid_b = -1;

@@ -163,6 +163,49 @@ __device__ __noinline__ void next_seq(const AttnTcParams& p, int lane, SeqWin& w
   }
 }
 
+// Warp-cooperative: pull the launch's lengths (ctx_lens, aux) into L2, one
+// 128-byte line per lane, so that the lookup after the dependency wait does
+// not pay DRAM latency for them.
+__device__ __forceinline__ void prefetch_lens_l2(const AttnTcParams& p, int lane) {
+  const int lines = (p.B * 4 + 127) / 128;
+  for (int i = lane; i < 2 * lines; i += 32) {
+    const int32_t* base = i < lines ? p.ctx_lens : p.aux;
+    const int li = i < lines ? i : i - lines;
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(base + li * 32) : "memory");
+  }
+}
+
+// ------------------------------------------------------------- merge plan
+// Entry c of the merge plan describes range boundary c (the first unit of
+// CTA c's range, c >= 1): when that boundary splits the tiles of a pair
+// (b, g) and is the first boundary to do so (CTA c - 1 holds the pair's first
+// tile), the entry is {b, g, slot of the first piece's record, c - 1, number
+// of pieces, query rows of the pair}; else b = -1.  CTA c writes it from the
+// lookup of its own range start, so that the merge kernel finds its pair with
+// one load instead of a scan of the cost line.  Lane 0 stores it; x, x1 are
+// the CTA's units, (b, g, t0, pc) what locate() gave for x and sq the
+// geometry of sequence b.
+__device__ __forceinline__ void write_merge_plan(const AttnTcParams& p, long long T, long long x,
+                                                 long long x1, int b, int g, int t0, long long pc,
+                                                 const SeqT& sq) {
+  const int c = (int)blockIdx.x;
+  if (c == 0) return;
+  int4 e0 = make_int4(-1, 0, 0, 0), e1 = make_int4(0, 0, 0, 0);
+  if (x < x1 && b < p.B && t0 > 0) {
+    const long long u0 = pc + kPairCost, u1 = u0 + sq.tiles - 1;
+    const int c_lo = cta_of(u0, T, p.nctas);
+    if (c_lo == c - 1) {
+      const int c_hi = cta_of(u1, T, p.nctas);
+      const int slot_lo = 2 * c_lo + (range_start(T, c_lo, p.nctas) >= pc ? 0 : 1);
+      e0 = make_int4(b, g, slot_lo, c_lo);
+      e1 = make_int4(c_hi - c_lo + 1, sq.nq * p.G, 0, 0);
+    }
+  }
+  int4* dst = reinterpret_cast<int4*>(p.plan + (size_t)c * kPlanInts);
+  dst[0] = e0;
+  dst[1] = e1;
+}
+
 // ------------------------------------------------------------- page boxes
 // Tensor maps of the paged cache for boxes of 1, 2, 4 and 8 consecutive pages
 // (64 head dims x 16 rows x 1 KV head x n pages): n pages whose ids follow one

@@ -269,8 +269,9 @@ __device__ __noinline__ void unit_epilogue(const AttnTcParams& p, int b, int g, 
 // attention kernel: the pieces' records are combined with weights
 // 2^(lse_i - M) / sum, in range order.  Block x looks at the boundary where
 // CTA x + 1's range starts and merges the pair that boundary splits, if it is
-// the pair's first such boundary; so the grid has one block column per
-// boundary, whatever the number of pairs.  One warp per query row (rows
+// the pair's first such boundary (the attention kernel's CTA x + 1 leaves
+// that in the merge plan); so the grid has one block column per boundary,
+// whatever the number of pairs.  One warp per query row (rows
 // 8 * blockIdx.y + warp), one lane per 4 head dims; each lane reads every
 // piece's log2-sum-exp and values in one online pass, kMergeBatch pieces at a
 // time.
@@ -294,71 +295,18 @@ template <> struct MergeVec<64> {
 
 template <int D>
 __global__ void __launch_bounds__(kMergeThreads) attn_merge_kernel(const AttnTcParams p) {
-  __shared__ long long sh_pc;
-  __shared__ int sh_b, sh_g;
   if (threadIdx.x == 0) pdl_trigger();
   pdl_wait();
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  // Block x handles range boundary c = x + 1 (the first unit of CTA c): the
-  // pair whose tiles that boundary splits, if any, and only when it is the
-  // first boundary inside the pair (CTA c - 1 holds the pair's first tile);
-  // so every shared pair is merged once and unshared pairs cost nothing.
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  // Block x handles range boundary c = x + 1: its plan entry, written by the
+  // attention kernel's CTA c, names the pair to merge (b < 0: none)
   const int c = blockIdx.x + 1;
-  // the cost line, block-parallel: thread i sums a contiguous chunk of
-  // sequences, a scan of the chunk sums gives T and each chunk's first unit,
-  // and the thread whose chunk holds unit x = start(c) walks it
-  __shared__ long long csum[kMergeThreads];
-  const int ch = (p.B + kMergeThreads - 1) / kMergeThreads;
-  const int b0 = tid * ch, b1 = min(p.B, b0 + ch);
-  long long mine = 0;
-  for (int i = b0; i < b1; ++i) mine += seq_cost(p, seq_of(p, i).tiles);
-  csum[tid] = mine;
-  if (tid == 0) sh_b = p.B;
-  __syncthreads();
-  for (int o = 1; o < kMergeThreads; o <<= 1) {   // inclusive scan
-    const long long v = tid >= o ? csum[tid - o] : 0;
-    __syncthreads();
-    csum[tid] += v;
-    __syncthreads();
-  }
-  const long long T = csum[kMergeThreads - 1];
-  const long long x = range_start(T, c, p.nctas);
-  long long base = csum[tid] - mine;
-  if (x < T && base <= x && x < csum[tid] && mine > 0) {
-    for (int i = b0; i < b1; ++i) {
-      const int tiles = seq_of(p, i).tiles;
-      const long long a = seq_cost(p, tiles);
-      if (x < base + a) {
-        const int per = tiles + kPairCost;
-        const int gg = (int)((x - base) / per);
-        const long long pc = base + (long long)gg * per;
-        const long long u0 = pc + kPairCost;
-        // the boundary splits the pair's tiles (x after its first tile) and
-        // is the first boundary to do so (CTA c - 1 holds the first tile)
-        if (x > u0 && cta_of(u0, T, p.nctas) == c - 1) {
-          sh_b = i;
-          sh_g = gg;
-          sh_pc = pc;
-        }
-        break;
-      }
-      base += a;
-    }
-  }
-  __syncthreads();
-  const int b = sh_b, g = sh_g;
-  if (b >= p.B) return;
-  const SeqT sq = seq_of(p, b);
+  const int4* pe = reinterpret_cast<const int4*>(p.plan + (size_t)c * kPlanInts);
+  const int4 e0 = __ldcg(pe), e1 = __ldcg(pe + 1);
+  const int b = e0.x, g = e0.y, slot_lo = e0.z, c_lo = e0.w;
+  const int nseg = e1.x, R = e1.y;
   const int r = blockIdx.y * kMergeRows + warp;   // query row j * G + head
-  if (sq.tiles == 0 || r >= sq.nq * p.G) return;
-  const long long pc = sh_pc;                      // the pair's first unit
-  const long long u0 = pc + kPairCost, u1 = u0 + sq.tiles - 1;         // its first and last tile
-  const int c_lo = cta_of(u0, T, p.nctas), c_hi = cta_of(u1, T, p.nctas);
-  if (c_lo == c_hi) return;
-  const int nseg = c_hi - c_lo + 1;
-  // the piece of CTA c_lo is its first piece unless the range of c_lo starts
-  // before the pair (then it holds the previous pair's last tile, unit pc - 1)
-  const int slot_lo = 2 * c_lo + (range_start(T, c_lo, p.nctas) >= pc ? 0 : 1);
+  if (b < 0 || r >= R) return;
   const int Rmax = p.G * p.W1;
   const size_t REC = (size_t)Rmax * (D + 1);
   using V = MergeVec<D>;
@@ -469,11 +417,10 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
   const int Rpad = (Rmax + 7) & ~7;
   const int nqb = Rpad <= 64 ? 2 : 1;
   const uint32_t qhalf = nqb == 2 ? (uint32_t)Rpad * 128u : kHalf;
-  // everything above touched only this CTA's shared and tensor memory
-  pdl_wait();
-
   if (warp == kWarpProducer) {
-    // ---------------------------------------------------------- producer
+    // descriptors are kernel parameters; the lengths are only pulled into L2
+    // (a prefetch returns nothing, so a predecessor still writing them is
+    // harmless): both before the dependency wait
     if (lane == 0) {
       tma_prefetch_desc(&tm_q);
       for (int i = 0; i < 4; ++i) {
@@ -485,6 +432,13 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
         tma_prefetch_desc(&tm_dv);
       }
     }
+    prefetch_lens_l2(p, lane);
+  }
+  // everything above touched only this CTA's shared and tensor memory
+  pdl_wait();
+
+  if (warp == kWarpProducer) {
+    // ---------------------------------------------------------- producer
     if (blockIdx.x == 0) {
       for (int b = lane; b < p.B; b += 32) {
         const int bad = seq_of(p, b).bad;
@@ -499,6 +453,10 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
     int b = p.B, g = 0, t0 = 0;
     long long pc = 0;   // first unit of pair (b, g)
     if (x < x1) locate(p, x, lane, win, b, g, t0, pc);
+    {
+      const SeqT s0 = b < p.B ? win_get(win, b) : SeqT{};
+      if (lane == 0) write_merge_plan(p, T, x, x1, b, g, t0, pc, s0);
+    }
     // K tiles in range order, each into the K ring as soon as a slot is free
     // (a slot frees when S of its tile is done).  Each tile's descriptor goes
     // to the descriptor ring, from which the V warp issues the tile's V.
@@ -1003,8 +961,17 @@ cudaError_t launch_attn_tc(const AttnTcParams& prm, const void* q, const void* k
   return launch_attn_merge(prm, kD, st);
 }
 
+size_t attn_tc_plan_offset(int32_t ctas, int32_t rows, int32_t head_dim) {
+  const size_t rec = 2 * (size_t)ctas * rows * (head_dim + 1) * sizeof(float);
+  return (rec + 15) & ~(size_t)15;
+}
+
+size_t attn_tc_records_bytes(int32_t ctas, int32_t rows, int32_t head_dim) {
+  return attn_tc_plan_offset(ctas, rows, head_dim) + (size_t)ctas * kPlanInts * sizeof(int32_t);
+}
+
 size_t attn_tc_part_bound(int32_t group, int32_t w1, int32_t head_dim) {
-  return 2 * (size_t)kTcMaxCtas * group * w1 * (head_dim + 1) * sizeof(float);
+  return attn_tc_records_bytes(kTcMaxCtas, group * w1, head_dim);
 }
 
 }  // namespace seedk

@@ -150,6 +150,7 @@ cudaError_t launch_f32_to_bf16(size_t n, const float* x, void* y, cudaStream_t s
 
 // Tensor-core draft and verify attention (attn_tc.cu).
 constexpr int kTcMaxCtas = 256;     // most CTAs of one launch (two record slots each)
+constexpr int kPlanInts = 8;        // int32 per merge plan entry
 
 struct AttnTcParams {
   const int32_t* page_table;
@@ -161,6 +162,7 @@ struct AttnTcParams {
   float* out;                 // f32 [B, W1, hq, 128]
   float* lse;                 // f32 [B, W1, hq] or null
   float* part;                // partial records: two slots per CTA
+  int32_t* plan;              // merge plan: 8 int32 per CTA range boundary
   int32_t* err;
   int32_t B, hq, hkv, kmax, G;
   int32_t draft;              // 1: draft attention (cache rows + draft scratch rows)
@@ -179,7 +181,12 @@ struct AttnTcParams {
 
 bool attn_tc_supported(int head_dim, int group, int w1);
 int attn_tc_ctas();
-// Workspace bytes of the split records of either tensor-core kernel.
+// Workspace of either tensor-core kernel, after its counters: two split
+// records per CTA (rows x (head_dim + 1) floats each), then, at
+// attn_tc_plan_offset, one 32-byte merge plan per CTA range boundary.
+size_t attn_tc_plan_offset(int32_t ctas, int32_t rows, int32_t head_dim);
+size_t attn_tc_records_bytes(int32_t ctas, int32_t rows, int32_t head_dim);
+// attn_tc_records_bytes at the most CTAs a launch uses.
 size_t attn_tc_part_bound(int32_t group, int32_t w1, int32_t head_dim);
 cudaError_t launch_attn_tc(const AttnTcParams& p, const void* q, const void* k_cache,
                            const void* v_cache, const void* draft_k, const void* draft_v,

@@ -102,7 +102,7 @@ seed_status_t run_attn_tc(const seed_cfg_t* cfg, int32_t batch, bool draft, cons
   const int W1 = draft ? 1 : cfg->kmax + 1;
   const size_t cb = kSchedBytes + counters_bytes(cfg, batch);
   const int ctas = seedk::attn_tc_ctas();
-  const size_t need = cb + 2 * (size_t)ctas * G * W1 * (cfg->head_dim + 1) * sizeof(float);
+  const size_t need = cb + seedk::attn_tc_records_bytes(ctas, G * W1, cfg->head_dim);
   const bool kt = seedk::attn_kt_supported(cfg->head_dim, G, W1);
   if (ws_bytes < need) return SEED_ERR_WORKSPACE;
   seedk::AttnTcParams p{};
@@ -115,6 +115,8 @@ seed_status_t run_attn_tc(const seed_cfg_t* cfg, int32_t batch, bool draft, cons
   p.out = out;
   p.lse = lse;
   p.part = reinterpret_cast<float*>(static_cast<char*>(ws) + cb);
+  p.plan = reinterpret_cast<int32_t*>(static_cast<char*>(ws) + cb +
+                                      seedk::attn_tc_plan_offset(ctas, G * W1, cfg->head_dim));
   p.err = err;
   p.B = batch;
   p.hq = cfg->hq;
