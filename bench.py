@@ -98,7 +98,8 @@ NCU_TRAFFIC = {
 }
 
 KERNEL_SOURCES = {
-    "attn_tc_kernel": ["attn_tc.cu", "tc.cuh", "common.cuh", "kernels.h"],
+    "attn_tc_kernel": ["attn_tc.cu", "attn_sched.cuh", "tc.cuh", "common.cuh", "kernels.h"],
+    "attn_kt_kernel": ["attn_kt.cu", "attn_sched.cuh", "tc.cuh", "common.cuh", "kernels.h"],
     "decode_attn_kernel": ["decode_attn.cu", "common.cuh", "kernels.h"],
 }
 
@@ -114,7 +115,7 @@ def kernel_source_hash(name: str) -> str:
 
 def ncu_traffic(wl, kind: str, alg_bytes: float):
     rec = NCU_TRAFFIC.get((wl.index, kind))
-    name = attn_kernel_name(wl)
+    name = attn_kernel_name(wl, kind)
     if rec is None or rec["kernel"] != name or rec["sources"] != kernel_source_hash(name):
         return None
     return round(rec["dram_bytes"] * alg_bytes / rec["alg_bytes"])
@@ -171,34 +172,83 @@ class ClockSampler:
 
 
 # ------------------------------------------------------------------ oracle leg
-def oracle_sample(wl, budget_s: float) -> dict:
-    """The oracle timed on host cores over a bounded sample of one round: the
-    draft attention of step 1 in both decoder layers and the verify attention
-    of as many layers as fit in the budget, all sequences."""
-    from oracle.workload import OracleRun
+def blas_threads():
+    """Threads of the BLAS that NumPy calls (the oracle's matrix products)."""
+    try:
+        from threadpoolctl import threadpool_info
+        n = [i.get("num_threads") for i in threadpool_info() if i.get("user_api") == "blas"]
+        if n:
+            return int(max(n))
+    except Exception:
+        pass
+    for k in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+        if os.environ.get(k, "").isdigit():
+            return int(os.environ[k])
+    return None
 
-    orc = OracleRun(wl, rounds=1)
-    lens = orc.lens.copy()
-    k_b = gen.round_plan(wl, 0)[0]
-    R = wl.row_bytes
-    qo = wl.hq * wl.head_dim * 6 + wl.hq * 4
-    done = 0
-    t0 = time.perf_counter()
-    for l in wl.dec_layers:
-        orc.draft(0, 1, l)
-        done += sum((int(L) + 1) * R + qo for L in lens)
-    layers = 0
-    while time.perf_counter() - t0 < budget_s and layers < wl.n_layers:
-        orc.verify(0, layers)
-        orc._ctx_cache.clear()
-        done += sum((int(L) + int(k) + 1) * R + (int(k) + 1) * qo for L, k in zip(lens, k_b))
-        layers += 1
-    dt = time.perf_counter() - t0
-    return {"value": done / dt / 1e9, "unit": UNIT, "cores": len(os.sched_getaffinity(0)),
-            "kind": "oracle", "seconds": round(dt, 2),
-            "sample": f"workload {wl.index}: draft step 1 in {len(wl.dec_layers)} decoder layers "
-                      f"+ verify attention of {layers} of {wl.n_layers} layers, all "
-                      f"{wl.batch} sequences, float64 NumPy"}
+
+class OracleSlice:
+    """A fixed slice of round 0 of the workload, run by the oracle on host
+    cores: draft step 1 in both decoder layers, then the verify attention of
+    layer 0, all sequences.  The same slice serves the reference arm (one
+    slice per step) and the cpu_baseline of the GPU arm (median of 3)."""
+
+    def __init__(self, wl):
+        from oracle.workload import OracleRun
+        self.wl = wl
+        self.orc = OracleRun(wl, rounds=1)
+        lens = self.orc.lens.copy()
+        k_b = gen.round_plan(wl, 0)[0]
+        R = wl.row_bytes
+        qo = wl.hq * wl.head_dim * 6 + wl.hq * 4
+        self.draft_bytes = len(wl.dec_layers) * sum((int(L) + 1) * R + qo for L in lens)
+        self.verify_bytes = sum((int(L) + int(k) + 1) * R + (int(k) + 1) * qo
+                                for L, k in zip(lens, k_b))
+        self.bytes = self.draft_bytes + self.verify_bytes
+        self.steps = int(k_b.max())
+
+    def run_draft(self) -> float:
+        t0 = time.perf_counter()
+        for l in self.wl.dec_layers:
+            self.orc.draft(0, 1, l)
+        return time.perf_counter() - t0
+
+    def run_verify(self) -> float:
+        t0 = time.perf_counter()
+        self.orc.verify(0, 0)
+        self.orc._ctx_cache.clear()
+        return time.perf_counter() - t0
+
+    def run(self) -> tuple[float, float]:
+        return self.run_draft(), self.run_verify()
+
+    def describe(self, td: float, tv: float, reps: int) -> dict:
+        wl = self.wl
+        t = td + tv
+        threads = blas_threads()
+        return {"value": self.bytes / t / 1e9, "unit": UNIT,
+                "cores": threads if threads else len(os.sched_getaffinity(0)),
+                "host_cores": len(os.sched_getaffinity(0)), "blas_threads": threads,
+                "kind": "oracle",
+                "sample": f"workload {wl.index}: draft step 1 in {len(wl.dec_layers)} decoder "
+                          f"layers + verify attention of 1 of {wl.n_layers} verify layers "
+                          f"(layer 0), all {wl.batch} sequences, float64 NumPy; "
+                          f"median of {reps}",
+                "slice_us": round(t * 1e6, 1),
+                "draft_layer_us": round(td * 1e6 / len(wl.dec_layers), 1),
+                "verify_layer_us": round(tv * 1e6, 1),
+                "round_us_extrapolated": round(
+                    1e6 * (td * self.steps + tv * wl.n_layers), 1),
+                "extrapolation": f"round = draft part x {self.steps} steps + verify layer x "
+                                 f"{wl.n_layers} layers (extrapolated, not timed)"}
+
+
+def oracle_sample(wl, reps: int = 3) -> dict:
+    """cpu_baseline: the fixed slice, timed reps times; the median slice."""
+    sl = OracleSlice(wl)
+    runs = sorted((sl.run() for _ in range(reps)), key=lambda x: x[0] + x[1])
+    td, tv = runs[len(runs) // 2]
+    return sl.describe(td, tv, reps)
 
 
 # ------------------------------------------------------------------ GPU leg
@@ -291,6 +341,7 @@ def run_seed(args, rank, world, device):
     t_round = [ev[t][0].elapsed_time(ev[t][3]) for t in range(K)]
     t_draft = [ev[t][0].elapsed_time(ev[t][1]) for t in range(K)]
     t_verify = [ev[t][1].elapsed_time(ev[t][2]) for t in range(K)]
+    t_accept = [ev[t][2].elapsed_time(ev[t][3]) for t in range(K)]
     byt = [round_bytes(wl, lens[W + t], gen.round_plan(wl, W + t)[0], len(dw.layers))
            for t in range(K)]
     total_ms = sum(t_round)
@@ -312,7 +363,8 @@ def run_seed(args, rank, world, device):
                           bytes=nbytes / launches, launches=launches)
 
     res = dict(total_ms=total_ms, total_bytes=total_bytes, t_round=t_round, t_draft=t_draft,
-               t_verify=t_verify, steps_per_round=steps_per_round, clocks=clocks, kern=kern,
+               t_verify=t_verify, t_accept=t_accept, steps_per_round=steps_per_round,
+               clocks=clocks, kern=kern,
                n_launches=count_launches(wl, steps_per_round, len(dw.layers)))
     if not args.no_e2e:
         res["e2e"] = run_e2e(dw, wl, stream, W, K, lens)
@@ -357,13 +409,18 @@ def attn_call_bytes(wl, kind, key, lens, k_b) -> int:
     return sum((int(L) + int(kb) + 1) * R + (int(kb) + 1) * qo for L, kb in zip(lens, k_b))
 
 
-def attn_kernel_name(wl) -> str:
-    """The kernel behind seed_draft_attn / seed_verify_attn for this shape: the
-    tensor-core kernel when head_dim is 128 and the query rows of one KV head
-    fit one 128-row tile, else the CUDA-core split-KV kernel."""
+def attn_kernel_name(wl, kind: str = "verify") -> str:
+    """The kernel behind seed_draft_attn / seed_verify_attn for this shape:
+    head_dim 128 with the query rows of one KV head in one 128-row tile: the
+    query-rows tensor-core kernel; head_dim 64 with at most 48 such rows: the
+    keys-as-rows tensor-core kernel; else the CUDA-core split-KV kernel."""
     G = wl.hq // wl.hkv
-    return "attn_tc_kernel" if wl.head_dim == 128 and G * (wl.kmax + 1) <= 128 \
-        else "decode_attn_kernel"
+    w1 = 1 if kind == "draft" else wl.kmax + 1
+    if wl.head_dim == 128 and G * w1 <= 128:
+        return "attn_tc_kernel"
+    if wl.head_dim == 64 and G * w1 <= 48:
+        return "attn_kt_kernel"
+    return "decode_attn_kernel"
 
 
 def run_profile(args):
@@ -435,9 +492,9 @@ def run_profile(args):
     assert int(dw.err.item()) == 0, f"device error flag {int(dw.err.item())} raised"
     key = (1, dec[0]) if args.profile == "draft" else dec[0]
     nbytes = attn_call_bytes(wl, "draft" if args.profile == "draft" else "verify", key, lens, k_b)
+    kname = attn_kernel_name(wl, "draft" if args.profile == "draft" else "verify")
     print(json.dumps({"profile": args.profile, "workload": wl.name,
-                      "kernel": attn_kernel_name(wl),
-                      "sources": kernel_source_hash(attn_kernel_name(wl)),
+                      "kernel": kname, "sources": kernel_source_hash(kname),
                       "alg_bytes_per_launch": nbytes,
                       "us": [round(ev[i].elapsed_time(ev[i + 1]) * 1e3, 1)
                              for i in range(args.reps)]}))
@@ -593,7 +650,7 @@ def run_profile_draftstep(args, wl):
 
 def run_profile_blockattn(args, wl, n=1000, block=10, batch=8):
     """--profile blockattn: the decoder's block-causal training attention
-    (Sec. 3) for `batch` sequences of n tokens in blocks of 10 (the paper's
+    (Sec. 4.2) for `batch` sequences of n tokens in blocks of 10 (the paper's
     training block size) at the workload's head shape, `--reps` calls back to
     back.  Reports the attention FLOPs (4 D per query head and visible key)
     against the bf16 peak and the bytes moved against the HBM peak: on the
@@ -761,6 +818,37 @@ def run_e2e(dw, wl, stream, W, K, lens):
             "d2h_bytes_per_step": d2h, "ms_per_step": ms / K}
 
 
+def per_workload(args, rank, device, peak) -> dict:
+    """Workloads 2, 3 and 5 (batch 1, a 16-sequence mix, the 64-sequence
+    paged mix), each from a fresh device workload: 3 warm-up and 3 timed
+    rounds, with the attention launches of 3 more rounds timed one by one."""
+    import copy
+    import torch
+    out = {}
+    for w in (2, 3, 5):
+        a = copy.copy(args)
+        a.workload, a.steps, a.warmup, a.no_e2e = w, 3, 3, True
+        r = run_seed(a, rank, 1, device)
+        wl = WORKLOADS[w]
+        kv_, kd_ = r["kern"]["verify"], r["kern"]["draft"]
+        out[str(w)] = {
+            "workload": wl.name,
+            "value": round(r["total_bytes"] / (r["total_ms"] / 1e3) / 1e9, 1), "unit": UNIT,
+            "round_us": round(1e3 * statistics.mean(r["t_round"]), 1),
+            "accept_us": round(1e3 * statistics.mean(r["t_accept"]), 2),
+            "verify": {"kernel": attn_kernel_name(wl), "us_per_launch": round(kv_["us"], 2),
+                       "achieved": round(kv_["gbs"], 1), "frac": round(kv_["gbs"] / peak, 3),
+                       "bytes_per_launch": round(kv_["bytes"]), "launches": kv_["launches"]},
+            "draft": {"kernel": attn_kernel_name(wl, "draft"), "us_per_launch": round(kd_["us"], 2),
+                      "achieved": round(kd_["gbs"], 1), "frac": round(kd_["gbs"] / peak, 3),
+                      "bytes_per_launch": round(kd_["bytes"]), "launches": kd_["launches"]},
+            "timing": "3 warm-up + 3 timed rounds; attention launches timed by CUDA events "
+                      "around each launch of 3 more rounds"}
+        del r
+        torch.cuda.empty_cache()
+    return out
+
+
 # ------------------------------------------------------------------ main
 def main():
     ap = argparse.ArgumentParser()
@@ -770,7 +858,10 @@ def main():
     ap.add_argument("--workload", type=int, default=4, choices=[1, 2, 3, 4, 5])
     ap.add_argument("--impl", default="seed", choices=["seed", "reference"])
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--cpu-budget", type=float, default=12.0)
+    ap.add_argument("--cpu-reps", type=int, default=3,
+                    help="timed repetitions of the oracle slice for cpu_baseline (0: none)")
+    ap.add_argument("--no-per-workload", action="store_true",
+                    help="skip the per-workload lines of workloads 2, 3 and 5")
     ap.add_argument("--profile", choices=["draft", "verify", "tree", "head", "draftstep",
                                           "blockattn"],
                     default=None,
@@ -799,19 +890,22 @@ def main():
     if args.impl == "reference":
         if rank != 0:
             return
-        vals = []
+        # one step = the oracle's fixed slice; a warm-up step runs its draft
+        # part (the oracle has no caches to warm, so that bounds the run)
+        sl = OracleSlice(wl)
         for _ in range(args.warmup):
-            oracle_sample(wl, min(args.cpu_budget, 3.0))
-        t0 = time.perf_counter()
-        for _ in range(args.steps):
-            vals.append(oracle_sample(wl, args.cpu_budget / max(1, args.steps)))
-        dt = time.perf_counter() - t0
-        v = statistics.mean(x["value"] for x in vals)
+            sl.run_draft()
+        runs = [sl.run() for _ in range(args.steps)]
+        runs.sort(key=lambda x: x[0] + x[1])
+        td, tv = runs[len(runs) // 2]
+        cpu = sl.describe(td, tv, args.steps)
+        v = cpu["value"]
         line = {"metric": METRIC, "value": v, "unit": UNIT, "impl": "reference", "n_gpus": 1,
                 "steps": args.steps, "warmup": args.warmup,
-                "ms_per_step": dt * 1e3 / args.steps, "higher_is_better": True, "scaling": "weak",
+                "ms_per_step": statistics.mean(a + b for a, b in runs) * 1e3,
+                "higher_is_better": True, "scaling": "weak",
                 "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": config,
-                "cpu_baseline": dict(vals[-1], value=v),
+                "cpu_baseline": cpu,
                 "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0,
                         "d2h_bytes_per_step": 0}}
         print(json.dumps(line))
@@ -825,7 +919,7 @@ def main():
 
     total_s, value = aggregate(res["total_bytes"], res["total_ms"] / 1e3, world, device)
     if rank == 0:
-        cpu = oracle_sample(wl, args.cpu_budget) if world == 1 else None
+        cpu = oracle_sample(wl, args.cpu_reps) if world == 1 and args.cpu_reps > 0 else None
         K = args.steps
         kv_, kd_ = res["kern"]["verify"], res["kern"]["draft"]
         line = {
@@ -838,6 +932,7 @@ def main():
             "draft_step_us": 1e3 * sum(res["t_draft"]) / sum(res["steps_per_round"]),
             "verify_step_us": 1e3 * statistics.mean(res["t_verify"]),
             "round_us": 1e3 * statistics.mean(res["t_round"]),
+            "accept_us": round(1e3 * statistics.mean(res["t_accept"]), 2),
             "roofline": {"bound": "hbm",
                          "kernel": f"seed_verify_attn ({attn_kernel_name(wl)})",
                          "achieved": round(kv_["gbs"], 1), "peak": peak,
@@ -847,7 +942,7 @@ def main():
                          "bytes_per_launch": round(kv_["bytes"]),
                          "us_per_launch": round(kv_["us"], 2), "launches": kv_["launches"],
                          "timing": "CUDA events around every launch of K more rounds"},
-            "draft_attn": {"kernel": f"seed_draft_attn ({attn_kernel_name(wl)})",
+            "draft_attn": {"kernel": f"seed_draft_attn ({attn_kernel_name(wl, "draft")})",
                            "achieved": round(kd_["gbs"], 1),
                            "frac": round(kd_["gbs"] / peak, 3),
                            "traffic": ncu_traffic(wl, "draft", kd_["bytes"]),
@@ -859,6 +954,8 @@ def main():
         }
         if "e2e" in res:
             line["e2e"] = res["e2e"]
+        if world == 1 and not args.no_per_workload:
+            line["per_workload"] = per_workload(args, rank, device, peak)
         print(json.dumps(line))
     if world > 1:
         torch.distributed.destroy_process_group()

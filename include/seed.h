@@ -403,7 +403,7 @@ seed_status_t seed_draft_layer(const seed_cfg_t* cfg, int32_t batch,
                                int32_t* err_flag, void* stream);
 
 /* ------------------------------------------------------------------------
- * The decoder's block-causal training attention (Sec. 3, "Training with
+ * The decoder's block-causal training attention (Sec. 4.2, "Training with
  * Block Attention"; Fig. 2, right), forward pass.  Sequences of n tokens are
  * cut into blocks of b; the query at position p sees
  *   - the deep keys/values k_dec/v_dec (the decoder layer's KV^dec from the
@@ -420,8 +420,9 @@ seed_status_t seed_draft_layer(const seed_cfg_t* cfg, int32_t batch,
  *   ws         seed_block_attn_workspace_bytes(...) bytes, 256-byte aligned,
  *              ZERO-FILLED before its first use.  head_dim 128 with 1, 2 or
  *              4 query heads per KV head runs one tensor-core kernel that
- *              reads q and the four inputs directly (the size is then 256
- *              and the workspace is not touched); other shapes run the
+ *              reads q and the four inputs directly (the size is then 256,
+ *              the workspace is not touched, and ws may be NULL with
+ *              ws_bytes 0); other shapes run the
  *              verify kernel on one virtual sequence per block, and the
  *              workspace holds its counters (every call leaves them zeroed)
  *              and a paged copy of the rows that each call rewrites.
@@ -453,8 +454,12 @@ seed_status_t seed_block_attn(const seed_cfg_t* cfg, int32_t batch, int32_t n, i
  *     SEED_NOALLOC_SCRATCH_BYTES.
  *   - Set-up: the first call on a device, with that device current, resolves
  *     the scratch's device address (this can load the library's module on
- *     the device) and caches it. Make that first call before any stream
- *     capture begins.
+ *     the device) and caches it with the id of the device's current context.
+ *   - Context changes: the scratch belongs to that context. When the device's
+ *     current context is a different one (after cudaDeviceReset, or with
+ *     another context made current), the next call resolves the address
+ *     again; nothing in the scratch carries over from one call to the next,
+ *     so no state is lost.
  *   - Zeroing: each call clears the scratch's counters on `stream` before its
  *     kernels (one small memset), so the caller never zeroes anything, and a
  *     call after a device error starts clean.

@@ -24,7 +24,7 @@ the paper (SEED: Self-Speculative Decoding via Implicit Encoder-Decoder):
   the pre-norm form of the paper's Qwen3 models (RMS norms, q/k norms, RoPE,
   grouped attention over the deep cache plus the draft rows, SwiGLU MLP),
   final norm and the dynamic-drafting head.
-* ``block_attn`` -- the decoder's block-causal training attention (Sec. 3,
+* ``block_attn`` -- the decoder's block-causal training attention (Sec. 4.2,
   "Training with Block Attention"; Fig. 2): deep-cache rows of the preceding
   blocks plus causal self-attention within the query's own block.
 * ``toy_model``  -- a tiny float64 transformer running Alg. 2 end to end (with

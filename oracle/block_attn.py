@@ -1,6 +1,6 @@
 """Block-causal training attention of the decoder (oracle; test infrastructure).
 
-Sec. 3 ("Training with Block Attention") trains the decoder for drafting by
+Sec. 4.2 ("Training with Block Attention") trains the decoder for drafting by
 cutting each sequence into blocks of b tokens.  In the decoder's pass over the
 raw embeddings H^0, the query at position p attends
 * to the decoder's deep cache KV^dec (from the full forward pass) at every

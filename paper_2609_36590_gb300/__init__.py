@@ -471,7 +471,7 @@ def seed_block_attn(cfg: SeedConfig, block: int, q, k_dec, v_dec, k_spec, v_spec
                     err, stream=None) -> None:
     """Block-causal training attention: q bf16 [B, n, hq, D]; k/v_dec and
     k/v_spec bf16 [B, n, hkv, D]; out f32 [B, n, hq, D]; lse f32 [B, n, hq]
-    or None."""
+    or None; ws uint8 (None on the tensor-core route, which uses none)."""
     B, n = q.shape[0], q.shape[1]
     kshape = (B, n, cfg.hkv, cfg.head_dim)
     c = cfg.c()
@@ -481,7 +481,8 @@ def seed_block_attn(cfg: SeedConfig, block: int, q, k_dec, v_dec, k_spec, v_spec
         _t(k_spec, torch.bfloat16, kshape, "k_spec"), _t(v_spec, torch.bfloat16, kshape, "v_spec"),
         _t(out, torch.float32, (B, n, cfg.hq, cfg.head_dim), "out"),
         _t(lse, torch.float32, (B, n, cfg.hq), "lse") if lse is not None else None,
-        _t(ws, torch.uint8, None, "ws"), ws.numel(), _t(err, torch.int32, (1,), "err"),
+        _t(ws, torch.uint8, None, "ws") if ws is not None else None,
+        ws.numel() if ws is not None else 0, _t(err, torch.int32, (1,), "err"),
         _stream(stream)))
 
 

@@ -166,12 +166,20 @@ __device__ __noinline__ void next_seq(const AttnTcParams& p, int lane, SeqWin& w
 // Warp-cooperative: pull the launch's lengths (ctx_lens, aux) into L2, one
 // 128-byte line per lane, so that the lookup after the dependency wait does
 // not pay DRAM latency for them.
+// A page table of at most 32 KiB is pulled in whole (the CTA's first pages
+// are not known before the lookup), a larger one not at all.
 __device__ __forceinline__ void prefetch_lens_l2(const AttnTcParams& p, int lane) {
   const int lines = (p.B * 4 + 127) / 128;
   for (int i = lane; i < 2 * lines; i += 32) {
     const int32_t* base = i < lines ? p.ctx_lens : p.aux;
     const int li = i < lines ? i : i - lines;
     asm volatile("prefetch.global.L2 [%0];" ::"l"(base + li * 32) : "memory");
+  }
+  const long long pt_bytes = (long long)p.B * p.max_pages * 4;
+  if (pt_bytes <= 32768) {
+    const int pl = (int)((pt_bytes + 127) / 128);
+    for (int i = lane; i < pl; i += 32)
+      asm volatile("prefetch.global.L2 [%0];" ::"l"(p.page_table + (size_t)i * 32) : "memory");
   }
 }
 

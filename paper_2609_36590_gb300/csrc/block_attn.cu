@@ -1,4 +1,4 @@
-// Block-causal training attention of the decoder (Sec. 3, "Training with
+// Block-causal training attention of the decoder (Sec. 4.2, "Training with
 // Block Attention"; Fig. 2): with blocks of b tokens, the query at position p
 // sees the decoder's deep keys/values (KV^dec) at positions < s(p) = (p/b)*b
 // and, causally, its own keys/values over the raw embeddings at positions
@@ -200,19 +200,19 @@ seed_status_t seed_block_attn(const seed_cfg_t* cfg, int32_t batch, int32_t n, i
   if (cfg == nullptr) return SEED_ERR_NULL;
   if (!block_ok(cfg, batch, n, block)) return SEED_ERR_SHAPE;
   if (batch == 0) return SEED_OK;
-  if (!q || !k_dec || !v_dec || !k_spec || !v_spec || !out || !ws || !err_flag)
-    return SEED_ERR_NULL;
+  if (!q || !k_dec || !v_dec || !k_spec || !v_spec || !out || !err_flag) return SEED_ERR_NULL;
   auto mis16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) != 0; };
   if (mis16(q) || mis16(k_dec) || mis16(v_dec) || mis16(k_spec) || mis16(v_spec) || mis16(out))
     return SEED_ERR_RANGE;
   if (seedk::block_tc_supported(cfg->head_dim, cfg->hq / cfg->hkv)) {
-    if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0 || ws_bytes < 256) return SEED_ERR_WORKSPACE;
+    // the tensor-core kernel uses no workspace: ws may be NULL, ws_bytes 0
     const float scale = cfg->scale > 0.f ? cfg->scale : 1.0f / std::sqrt((float)cfg->head_dim);
     const cudaError_t e = seedk::launch_block_tc(batch, n, block, cfg->hq, cfg->hkv, scale, q,
                                                  k_dec, v_dec, k_spec, v_spec, out, lse,
                                                  err_flag, static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? SEED_OK : SEED_ERR_CUDA;
   }
+  if (ws == nullptr) return SEED_ERR_NULL;
   const BlockGeom g = geom(batch, n, block, cfg->hkv, cfg->head_dim);
   if (g.num_pages > INT32_MAX) return SEED_ERR_SHAPE;
   const seed_cfg_t v = virtual_cfg(cfg, block);

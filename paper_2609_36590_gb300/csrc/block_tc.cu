@@ -1,4 +1,4 @@
-// Block-causal training attention on the tensor cores (Sec. 3, "Training
+// Block-causal training attention on the tensor cores (Sec. 4.2, "Training
 // with Block Attention"; Fig. 2): the query at position p sees the deep rows
 // KV^dec at positions < s(p) = (p / b) * b and its own block's raw-embedding
 // rows at positions s(p) .. p.

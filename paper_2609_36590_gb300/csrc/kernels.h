@@ -181,6 +181,13 @@ struct AttnTcParams {
 
 bool attn_tc_supported(int head_dim, int group, int w1);
 int attn_tc_ctas();
+// Bytes at the start of a draft / verify workspace that must be zero before
+// a call (every kernel leaves them zero again): 256 bytes of work-dispenser
+// state, then one int32 arrival counter per (sequence, query slot, KV head)
+// with at least 4 slots per sequence, rounded up to 256 bytes.  The rest of
+// the workspace holds split records and plans, always written before read.
+size_t workspace_zero_prefix_bytes(int32_t kmax, int32_t hkv, int32_t batch);
+
 // Workspace of either tensor-core kernel, after its counters: two split
 // records per CTA (rows x (head_dim + 1) floats each), then, at
 // attn_tc_plan_offset, one 32-byte merge plan per CTA range boundary.

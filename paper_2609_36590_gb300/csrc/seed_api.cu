@@ -15,6 +15,19 @@ constexpr size_t kAlign = 256;
 
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
+}  // namespace
+
+namespace seedk {
+
+size_t workspace_zero_prefix_bytes(int32_t kmax, int32_t hkv, int32_t batch) {
+  const size_t per = (size_t)std::max(kmax + 1, 4);
+  return kAlign + round_up((size_t)batch * per * hkv * sizeof(int32_t), kAlign);
+}
+
+}  // namespace seedk
+
+namespace {
+
 bool group_supported(int g) { return g == 1 || g == 2 || g == 4 || g == 8; }
 
 seed_status_t check_cfg(const seed_cfg_t* cfg) {
@@ -42,11 +55,11 @@ float scale_of(const seed_cfg_t* cfg) {
 // Workspace layout: [0, 256) the tensor-core verify's unit dispenser; then
 // arrival counters for batch*(kmax+1)*hkv (virtual sequence, KV head) pairs;
 // then the split partial records.  Every kernel leaves the counters at zero.
+// The first two parts are the zero prefix (seedk::workspace_zero_prefix_bytes).
 constexpr size_t kSchedBytes = kAlign;
 
-size_t counters_bytes(const seed_cfg_t* cfg, int32_t batch) {
-  const size_t per = std::max(cfg->kmax + 1, 4);
-  return round_up((size_t)batch * per * cfg->hkv * sizeof(int32_t), kAlign);
+size_t zero_prefix(const seed_cfg_t* cfg, int32_t batch) {
+  return seedk::workspace_zero_prefix_bytes(cfg->kmax, cfg->hkv, batch);
 }
 
 seed_status_t finish(cudaError_t e) { return e == cudaSuccess ? SEED_OK : SEED_ERR_CUDA; }
@@ -59,7 +72,7 @@ seed_status_t run_decode(const seed_cfg_t* cfg, int32_t batch, bool verify, cons
   const int nq = verify ? cfg->kmax + 1 : 1;
   const int nv = batch * nq;
   const seedk::DecodePlan pl = seedk::plan_decode(nv, cfg->hkv, G, cfg->head_dim, kv.max_pages);
-  const size_t cb = kSchedBytes + counters_bytes(cfg, batch);
+  const size_t cb = zero_prefix(cfg, batch);
   if (ws_bytes < cb + pl.part_bytes) return SEED_ERR_WORKSPACE;
   seedk::DecodeParams p{};
   p.q = static_cast<const uint16_t*>(q);
@@ -100,7 +113,7 @@ seed_status_t run_attn_tc(const seed_cfg_t* cfg, int32_t batch, bool draft, cons
                           const uint32_t* anc = nullptr) {
   const int G = cfg->hq / cfg->hkv;
   const int W1 = draft ? 1 : cfg->kmax + 1;
-  const size_t cb = kSchedBytes + counters_bytes(cfg, batch);
+  const size_t cb = zero_prefix(cfg, batch);
   const int ctas = seedk::attn_tc_ctas();
   const size_t need = cb + seedk::attn_tc_records_bytes(ctas, G * W1, cfg->head_dim);
   const bool kt = seedk::attn_kt_supported(cfg->head_dim, G, W1);
@@ -177,7 +190,7 @@ size_t seed_workspace_bytes(const seed_cfg_t* cfg, int32_t batch) {
     part = std::max(part, seedk::attn_tc_part_bound(G, 1, cfg->head_dim));
   if (tc_path(cfg->head_dim, G, cfg->kmax + 1))
     part = std::max(part, seedk::attn_tc_part_bound(G, cfg->kmax + 1, cfg->head_dim));
-  return kSchedBytes + counters_bytes(cfg, batch) + round_up(part, kAlign);
+  return zero_prefix(cfg, batch) + round_up(part, kAlign);
 }
 
 seed_status_t seed_draft_kv_append(const seed_cfg_t* cfg, int32_t batch, const void* k_new,

@@ -236,10 +236,13 @@ def test_block_attn_host_checks(lib):
     assert call(cf=_Cfg(32, 8, 96, 16, 8, 0.0)) == ERR_SHAPE
     assert call(q=None) == ERR_NULL
     assert call(q=FAKE + 8) == ERR_RANGE
-    assert call(nbytes=128) == ERR_WS              # tensor-core route: 256 bytes
-    assert call(ws=FAKE + 16) == ERR_WS
+    # the tensor-core route (head_dim 128, groups 1-4) takes no workspace, so
+    # its ws checks are gone (and a valid call would launch: none is made
+    # here); the virtual-sequence route still checks it
     c64 = _Cfg(32, 8, 64, 16, 8, 0.0)            # head_dim 64: the virtual-sequence route
     assert call(cf=c64, nbytes=4096) == ERR_WS
+    assert call(cf=c64, ws=FAKE + 16) == ERR_WS
+    assert call(cf=c64, ws=None) == ERR_NULL
     assert lib.seed_block_attn_workspace_bytes(ctypes.byref(c64), 2, 40, 10) > 4096
     assert lib.seed_block_attn_workspace_bytes(ctypes.byref(c), 2, 40, 10) == 256
     assert lib.seed_block_attn_workspace_bytes(ctypes.byref(c), 2, 41, 10) == 0

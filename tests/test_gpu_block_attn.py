@@ -1,11 +1,15 @@
-"""GPU parity of the decoder's block-causal training attention (Sec. 3,
+"""GPU parity of the decoder's block-causal training attention (Sec. 4.2,
 "Training with Block Attention"; Fig. 2) through the C ABI against the
 oracle: o and lse within the attention tolerance (max abs <= 2e-3, max rel
 <= 1e-2 on |o| > 1e-2) for block sizes 2 to 32, head_dim 64 and 128, group
 sizes 1 to 4, block boundaries inside and across 16-row pages and 128-row
 key tiles, query tiles cut by the sequence end; a 4B-shaped
-sequence pair of 1000 tokens in blocks of 10 on sampled positions; and the
-workspace left reusable (a second call on it gives the same result)."""
+sequence pair of 1000 tokens in blocks of 10 on sampled positions; the
+workspace left reusable (a second call on it gives the same result); and on
+the tensor-core route (called without a workspace), key rows that push a
+row's maximum up by more than 2^8 in later key tiles (1 % of rows scaled by
+8, or a low first tile followed by large keys), which exercises the
+kernel's rescale of its accumulator."""
 
 import numpy as np
 import pytest
@@ -46,15 +50,21 @@ def close(got, ref, what):
         assert (diff[big] / np.abs(ref[big])).max() <= RTOL, what
 
 
-def run(S, B, n, b, hq, hkv, D, seed):
+def run(S, B, n, b, hq, hkv, D, seed, keys=None, ws=True):
+    """keys(g, k_dec, k_spec) -> (k_dec, k_spec): optional reshaping of the
+    key rows (float32) before they are rounded to bf16."""
     g = np.random.default_rng(seed)
     qb = bits(g, (B, n, hq, D))
     kv = [bits(g, (B, n, hkv, D)) for _ in range(4)]
+    if keys is not None:
+        f32 = gen.bf16_bits_to_f32
+        kd, ks = keys(g, f32(kv[0]).copy(), f32(kv[2]).copy())
+        kv[0], kv[2] = gen.f32_to_bf16_bits(kd), gen.f32_to_bf16_bits(ks)
     cfg = S.SeedConfig(hq=hq, hkv=hkv, head_dim=D, kmax=1)
     out = torch.full((B, n, hq, D), 7.0, device="cuda")
     lse = torch.full((B, n, hq), 7.0, device="cuda")
     err = torch.zeros(1, dtype=torch.int32, device="cuda")
-    ws = S.new_block_attn_workspace(cfg, B, n, b)
+    ws = S.new_block_attn_workspace(cfg, B, n, b) if ws else None
     S.seed_block_attn(cfg, b, dev16(qb), *[dev16(x) for x in kv], out, lse, ws, err)
     torch.cuda.synchronize()
     assert int(err.item()) == 0
@@ -114,3 +124,53 @@ def test_block_attn_4b_shape_sampled(S):
     S.seed_block_attn(cfg, b, dev16(qb), *[dev16(x) for x in kv], out2, None, ws, err)
     torch.cuda.synchronize()
     np.testing.assert_array_equal(out2.cpu().numpy(), out.astype(np.float32))
+
+
+def stress_keys(frac):
+    """About frac of the key rows (decoder and speculative) scaled by 8: their
+    scores jump far above the running maximum in whatever key tile they
+    fall, so the softmax's rescale of O runs in later tiles."""
+    def f(g, kd, ks):
+        for k in (kd, ks):
+            rows = g.random(k.shape[:2]) < frac
+            k[rows] *= 8.0
+        return kd, ks
+    return f
+
+
+def low_then_high(g, kd, ks):
+    """Decoder rows of the first 128 positions (the first deep key tile)
+    scaled by 1/16, later ones by 4: a row's maximum over the first tile is
+    exceeded by far more than 2^8 in later tiles."""
+    kd[:, :128] *= 1.0 / 16.0
+    kd[:, 128:] *= 4.0
+    return kd, ks
+
+
+# B, n, b, hq, hkv, D on the tensor-core route (head_dim 128, groups 1, 2, 4),
+# several key tiles per item
+RESCALE_CASES = [
+    (1, 400, 10, 8, 8, 128, "stress"),
+    (1, 400, 10, 8, 4, 128, "stress"),
+    (2, 304, 16, 16, 4, 128, "stress"),
+    (1, 520, 8, 8, 2, 128, "low_then_high"),
+    (1, 400, 20, 4, 4, 128, "low_then_high"),
+]
+
+
+@pytest.mark.parametrize("case", RESCALE_CASES,
+                         ids=lambda c: "B{}_n{}_b{}_h{}x{}_D{}_{}".format(*c))
+def test_block_attn_rescale_matches_oracle(S, case):
+    """Later key tiles whose scores exceed the running maximum by more than
+    2^8: the tensor-core kernel rescales its O accumulator (softmax attention
+    does not depend on the reference maximum m in 2^(s_j - m), so the result
+    must match the oracle whatever m the kernel holds)."""
+    B, n, b, hq, hkv, D, kind = case
+    keys = stress_keys(0.01) if kind == "stress" else low_then_high
+    qb, kv, out, lse, _ = run(S, B, n, b, hq, hkv, D, seed=sum(case[:6]) + 7, keys=keys,
+                              ws=False)
+    f = gen.bf16_bits_to_f64
+    for s in range(B):
+        o, l = OB.block_causal_attention(f(qb[s]), *(f(x[s]) for x in kv), b, OAT.default_scale(D))
+        close(out[s], o, f"o seq {s}")
+        close(lse[s], l, f"lse seq {s}")

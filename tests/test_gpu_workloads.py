@@ -2,7 +2,8 @@
 bench times (one C-ABI call per layer and draft step): the tiny check and the
 4B batch-1 shape in full; batch 16, the 32k-token stress case and the 32-round
 paged serving mix on sampled layers and sequences, computed one by one by the
-oracle.  Accepted lengths, tokens, committed slots and lengths: bit-exact every
+oracle; in the serving mix, every rolled-back cache slot is overwritten with
+NaN after each accept, so a read of one would show as a non-finite output.  Accepted lengths, tokens, committed slots and lengths: bit-exact every
 round.  Attention: max abs <= 2e-3, max rel <= 1e-2 (|o| > 1e-2)."""
 
 import numpy as np
@@ -37,15 +38,39 @@ def DW():
     return DeviceWorkload
 
 
-def run_and_check(DW, idx, layers=None, rounds=None, sample_b=None, verify_layers=None):
+def poison_rolled_back(dw, lens_before, k_b):
+    """Write bf16 NaN into every cache slot that the round's verify appended
+    and the accept rolled back (positions L + n + 1 .. L + k_b of each
+    sequence, in every materialised layer), so that any later read of a
+    rolled-back row would turn that output into NaN (Alg. 2: only the
+    accepted prefix is committed)."""
+    acc = dw.accepted.cpu().numpy()
+    n = 0
+    for b in range(len(lens_before)):
+        lo, hi = int(lens_before[b]) + int(acc[b]) + 1, int(lens_before[b]) + int(k_b[b])
+        if hi < lo:
+            continue
+        pos = np.arange(lo, hi + 1)
+        pages = torch.from_numpy(dw.pt_np[b, pos // 16].astype(np.int64)).to(dw.device)
+        slots = torch.from_numpy((pos % 16).astype(np.int64)).to(dw.device)
+        for l in dw.layers:
+            dw.kv[l].k[pages, :, slots] = float("nan")
+            dw.kv[l].v[pages, :, slots] = float("nan")
+        n += len(pos)
+    return n
+
+
+def run_and_check(DW, idx, layers=None, rounds=None, sample_b=None, verify_layers=None,
+                  poison=False):
     """Run the workload's rounds on the GPU; check every accept bit-exactly and
-    the attention outputs of the sampled (layer, sequence) pairs."""
+    the attention outputs of the sampled (layer, sequence) pairs.  poison:
+    after every accept, NaN into the rolled-back slots (poison_rolled_back)."""
     wl = WORKLOADS[idx]
     n_rounds = wl.rounds if rounds is None else rounds
     dw = DW(wl, layers=layers, rounds=n_rounds)
     orc = OracleRun(wl, rounds=n_rounds)
     np.testing.assert_array_equal(orc.page_table, dw.pt_np)
-    checked = 0
+    checked = poisoned = 0
     for rnd in range(n_rounds):
         bs = list(range(wl.batch)) if sample_b is None else sample_b(rnd)
         vl = dw.layers if verify_layers is None else verify_layers(rnd)
@@ -58,6 +83,7 @@ def run_and_check(DW, idx, layers=None, rounds=None, sample_b=None, verify_layer
             if l in vl:
                 got_v[l] = (out[bs].cpu().numpy(), lse[bs].cpu().numpy())
 
+        lens_before = dw.ctx_lens.cpu().numpy().copy()
         dw.run_round(rnd, on_draft=on_draft, on_verify=on_verify)
         torch.cuda.synchronize()
         assert int(dw.err.item()) == 0, f"device error flag {int(dw.err.item())}"
@@ -82,8 +108,11 @@ def run_and_check(DW, idx, layers=None, rounds=None, sample_b=None, verify_layer
         np.testing.assert_array_equal(dw.tokens.cpu().numpy(), tok)
         np.testing.assert_array_equal(dw.slots.cpu().numpy(), slots)
         np.testing.assert_array_equal(dw.ctx_lens.cpu().numpy(), new_lens)
+        if poison:
+            poisoned += poison_rolled_back(dw, lens_before, dw.round_inputs(rnd)["k_b_np"])
         orc._ctx_cache.clear()
     assert checked > 0
+    assert poisoned > 0 or not poison
     return dw, orc
 
 
@@ -109,5 +138,5 @@ def test_workload5_serving_mix_32_rounds(DW):
     picks = [sorted(rng.choice(wl.batch, size=3, replace=False).tolist()) for _ in range(wl.rounds)]
     layers = [3, 11, 26, 27]
     dw, orc = run_and_check(DW, 5, layers=layers, sample_b=lambda r: picks[r],
-                            verify_layers=lambda r: [layers[r % 2], 26, 27])
+                            verify_layers=lambda r: [layers[r % 2], 26, 27], poison=True)
     assert (orc.lens > orc.lens0).all()

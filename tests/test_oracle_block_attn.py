@@ -1,4 +1,4 @@
-"""Pins of the block-causal training attention oracle (Sec. 3, "Training with
+"""Pins of the block-causal training attention oracle (Sec. 4.2, "Training with
 Block Attention"; Fig. 2), against things other than itself:
 * the mask of Fig. 2 (n = 6, b = 2) worked by hand (tests/golden);
 * the paper's 1-based boundary n' = floor((j - 2) / b) * b + 1 for every

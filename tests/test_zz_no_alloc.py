@@ -8,7 +8,10 @@ gets the same status as seed_verify_attn.
 GPU side: through the C ABI, two calls in a row match seed_verify_attn (with
 its own zero-filled workspace) within the parity tolerance, on tensor-core
 and CUDA-core shapes with split units, and the second call changes the
-device's free memory by nothing.  The file is named to be collected last, so
+device's free memory by nothing.  One shape is also checked against the
+oracle (Sec. 4.1 verify attention), and a call whose lengths the kernel
+rejects (SEED_DEVERR_CTX_LEN) leaves the scratch fit for the next, valid
+call, which again matches the oracle.  The file is named to be collected last, so
 that it also runs after every other test in one process.
 """
 
@@ -23,6 +26,7 @@ from workloads import gen
 ATOL, RTOL = 2e-3, 1e-2
 SENTINEL = 12345.0
 FAKE = 0x10000  # never dereferenced: the calls that use it fail a host check first
+DEVERR_CTX_LEN = 1  # SEED_DEVERR_CTX_LEN of include/seed.h
 
 
 @pytest.fixture(scope="module")
@@ -67,13 +71,15 @@ def test_invalid_cfg_and_empty_batch(lib):
 
 
 # B, hq, hkv, D, kmax, max_ctx: long enough contexts that pairs split into
-# several units (the arrival counters in the scratch are used), one D=64
-# shape on the CUDA-core kernel, and the largest kmax.
+# several units (the arrival counters in the scratch are used), a D=64 shape
+# on the keys-as-rows kernel (20 query rows per KV head), one on the
+# CUDA-core kernel (72 rows), and the largest kmax.
 CASES = [
     (6, 32, 8, 128, 4, 3000),
     (5, 32, 8, 128, 8, 1100),
     (4, 16, 16, 128, 16, 700),
     (7, 8, 2, 64, 4, 2500),
+    (5, 16, 2, 64, 8, 2500),
 ]
 
 
@@ -147,3 +153,63 @@ def test_noalloc_matches_workspace_entry_point(lib, case):
             if n:
                 assert_close(o[b, :n], ref_o[b, :n], f"call {i} out b={b}")
                 assert_close(l[b, :n], ref_l[b, :n], f"call {i} lse b={b}")
+
+
+def setup_case(S, seed, B, hq, hkv, D, kmax, max_ctx):
+    c = gen.small_case(seed, B, hq, hkv, D, kmax, max_ctx, True, 1.0)
+    cfg = S.SeedConfig(hq=hq, hkv=hkv, head_dim=D, kmax=kmax)
+    num_pages = B * c["max_pages"]
+    nrows = c["lens"] + c["n_q"]
+    kv = S.PagedKV(dev16(paged(c["rows_k"], nrows, c["page_table"], num_pages)),
+                   dev16(paged(c["rows_v"], nrows, c["page_table"], num_pages)),
+                   torch.from_numpy(c["page_table"]).cuda())
+    return c, cfg, kv
+
+
+def check_against_oracle(c, o, l, D, what):
+    from oracle import attention as OAT
+    f64 = gen.bf16_bits_to_f64
+    for b in range(len(c["lens"])):
+        n, L = int(c["n_q"][b]), int(c["lens"][b])
+        assert (o[b, n:] == SENTINEL).all() and (l[b, n:] == SENTINEL).all()
+        if n == 0:
+            continue
+        ro, rl = OAT.verify_attention_seq(f64(c["q_verify"][b, :n]), f64(c["rows_k"][b, :L + n]),
+                                          f64(c["rows_v"][b, :L + n]), L, OAT.default_scale(D))
+        assert_close(o[b, :n], ro, f"{what} out b={b} L={L} n={n}")
+        assert_close(l[b, :n], rl, f"{what} lse b={b}")
+
+
+@pytest.mark.gpu
+def test_noalloc_matches_oracle_and_recovers_after_a_rejected_call(lib):
+    assert torch.cuda.is_available(), "GPU test run without a GPU"
+    import paper_2609_36590_gb300 as S
+    B, hq, hkv, D, kmax, max_ctx = 6, 32, 8, 128, 4, 3000
+    c, cfg, kv = setup_case(S, 37, B, hq, hkv, D, kmax, max_ctx)
+    q = dev16(c["q_verify"])
+    n_q = torch.from_numpy(c["n_q"]).cuda()
+    W = kmax + 1
+
+    def call(lens_np):
+        o = torch.full((B, W, hq, D), SENTINEL, device="cuda")
+        l = torch.full((B, W, hq), SENTINEL, device="cuda")
+        e = torch.zeros(1, dtype=torch.int32, device="cuda")
+        S.seed_verify_attn_noalloc(cfg, q, n_q, kv, torch.from_numpy(lens_np).cuda(), o, l, e)
+        torch.cuda.synchronize()
+        return o.cpu().numpy(), l.cpu().numpy(), int(e.item())
+
+    o, l, e = call(c["lens"])
+    assert e == 0
+    check_against_oracle(c, o, l, D, "noalloc")
+
+    # lengths past the page table's capacity: the kernels' host-independent
+    # checks reject those sequences (no row is read for them) and flag it
+    bad = c["lens"].copy()
+    bad[0] = kv.page_table.shape[1] * 16
+    bad[2] = kv.page_table.shape[1] * 16 + 5
+    _, _, e = call(bad)
+    assert e & DEVERR_CTX_LEN
+
+    o, l, e = call(c["lens"])
+    assert e == 0, f"device error {e} after a rejected call"
+    check_against_oracle(c, o, l, D, "noalloc after rejected call")
