@@ -91,10 +91,10 @@ def round_bytes(wl, lens: np.ndarray, k_b: np.ndarray, n_layers: int) -> dict:
 # reported traffic is scaled to the timed launches by their algorithmic bytes,
 # and is null once the kernel's sources differ from the captured ones.
 NCU_TRAFFIC = {
-    (4, "verify"): {"kernel": "attn_tc_kernel", "sources": "e62147c3b201117d",
-                    "dram_bytes": 538025728 + 10420480, "alg_bytes": 537907712},
-    (4, "draft"): {"kernel": "attn_tc_kernel", "sources": "e62147c3b201117d",
-                   "dram_bytes": 537406720 + 10487040, "alg_bytes": 536986112},
+    (4, "verify"): {"kernel": "attn_tc_kernel", "sources": "540ecf203b3abbd1",
+                    "dram_bytes": 537898752 + 3558144, "alg_bytes": 537907712},
+    (4, "draft"): {"kernel": "attn_tc_kernel", "sources": "540ecf203b3abbd1",
+                   "dram_bytes": 537406720 + 3299328, "alg_bytes": 536986112},
 }
 
 KERNEL_SOURCES = {
@@ -439,6 +439,17 @@ def run_profile(args):
     from workloads.device import DeviceWorkload
 
     wl = WORKLOADS[args.workload]
+    if args.prefix is not None or args.batch is not None:
+        # the workload's heads and draft lengths with a fixed prefix length
+        # and/or another batch (e.g. a head_dim 64 verify over a 32k prefix)
+        import dataclasses
+        L = args.prefix if args.prefix is not None else wl.ctx_lo
+        B = args.batch if args.batch is not None else wl.batch
+        fixed = args.prefix is not None
+        wl = dataclasses.replace(wl, batch=B, ctx="fixed" if fixed else wl.ctx,
+                                 ctx_lo=L if fixed else wl.ctx_lo,
+                                 ctx_hi=L if fixed else wl.ctx_hi,
+                                 name=f"{wl.name} (batch {B}, prefix {L if fixed else 'as is'})")
     torch.cuda.set_device(0)
     if args.profile == "head":
         run_profile_head(args, wl, args.head_batch)
@@ -867,6 +878,11 @@ def main():
                     default=None,
                     help="launch one attention kind a few times for an ncu capture")
     ap.add_argument("--reps", type=int, default=3)
+    ap.add_argument("--prefix", type=int, default=None,
+                    help="--profile draft|verify|tree: a fixed prefix length instead of the "
+                         "workload's")
+    ap.add_argument("--batch", type=int, default=None,
+                    help="--profile draft|verify|tree: batch instead of the workload's")
     ap.add_argument("--head-batch", type=int, default=None,
                     help="--profile head: batch instead of the workload's")
     args = ap.parse_args()

@@ -145,6 +145,46 @@ __device__ __noinline__ void locate(const AttnTcParams& p, long long x, int lane
   pc = 0;
 }
 
+// Warp-cooperative: this CTA's units [x, x1) of the T units of the launch, and
+// (when x < x1) what locate() gives for x.  Up to 32 sequences the lengths
+// are loaded once: the lanes keep their sequence's geometry from the total
+// and find x in it; larger batches take total_cost() and locate().
+__device__ __noinline__ void lookup_range(const AttnTcParams& p, int lane, long long& T,
+                                          long long& x, long long& x1, SeqWin& w, int& b, int& g,
+                                          int& t, long long& pc) {
+  const int c = (int)blockIdx.x;
+  b = p.B;
+  g = t = 0;
+  pc = 0;
+  if (p.B > 32) {
+    T = total_cost(p, lane);
+    x = range_start(T, c, p.nctas);
+    x1 = range_start(T, c + 1, p.nctas);
+    if (x < x1) locate(p, x, lane, w, b, g, t, pc);
+    return;
+  }
+  w.wb = 0;
+  w.mine = seq_or_empty(p, lane);
+  const long long a = seq_cost(p, w.mine.tiles);
+  long long inc = a;
+  for (int o = 1; o < 32; o <<= 1) {
+    const long long v = __shfl_up_sync(kFull, inc, o);
+    if (lane >= o) inc += v;
+  }
+  T = __shfl_sync(kFull, inc, 31);
+  x = range_start(T, c, p.nctas);
+  x1 = range_start(T, c + 1, p.nctas);
+  if (x >= x1) return;
+  const unsigned m = __ballot_sync(kFull, inc - a <= x && x < inc);
+  const int src = __ffs(m) - 1;
+  const long long sb = __shfl_sync(kFull, inc - a, src);
+  const int per = __shfl_sync(kFull, w.mine.tiles, src) + kPairCost;
+  b = src;
+  g = (int)((x - sb) / per);
+  pc = sb + (long long)g * per;
+  t = (int)max(0LL, x - pc - kPairCost);
+}
+
 // Warp-cooperative: the next sequence after b with at least one tile (p.B if
 // none), moving the window forward as needed.
 __device__ __noinline__ void next_seq(const AttnTcParams& p, int lane, SeqWin& w, int& b) {

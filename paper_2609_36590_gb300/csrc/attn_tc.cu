@@ -446,13 +446,11 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
       }
     }
     // this CTA's units [x, x1)
-    const long long T = total_cost(p, lane);
-    const long long x = range_start(T, blockIdx.x, p.nctas);
-    const long long x1 = range_start(T, blockIdx.x + 1, p.nctas);
+    long long T, x, x1;
     SeqWin win;
     int b = p.B, g = 0, t0 = 0;
     long long pc = 0;   // first unit of pair (b, g)
-    if (x < x1) locate(p, x, lane, win, b, g, t0, pc);
+    lookup_range(p, lane, T, x, x1, win, b, g, t0, pc);
     {
       const SeqT s0 = b < p.B ? win_get(win, b) : SeqT{};
       if (lane == 0) write_merge_plan(p, T, x, x1, b, g, t0, pc, s0);
