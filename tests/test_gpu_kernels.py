@@ -64,6 +64,10 @@ CASES = [
     (4, 16, 16, 128, 16, 200, True, 1.0),
     (4, 16, 8, 64, 2, 500, True, 8.0),
     (3, 64, 8, 128, 4, 100, True, 1.0),
+    # few (sequence, KV head) pairs with long contexts: each pair split over
+    # many CTAs, G = 8 query heads per KV head
+    (9, 8, 1, 128, 4, 3000, True, 1.0),
+    (16, 8, 1, 128, 8, 1100, True, 1.0),
 ]
 
 

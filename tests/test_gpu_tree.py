@@ -85,6 +85,8 @@ TREE_CASES = [
     (4, 32, 8, 128, 31, 1100, False),
     (5, 16, 16, 128, 12, 2000, True),
     (3, 64, 8, 128, 15, 500, True),
+    (9, 8, 1, 128, 7, 3000, True),     # few pairs, long contexts: pairs split over many CTAs
+    (6, 8, 4, 64, 7, 500, True),       # head_dim 64, 16 rows: the keys-as-rows kernel
 ]
 
 
