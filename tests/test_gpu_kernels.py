@@ -288,8 +288,10 @@ def test_accept_commit_is_bit_exact(S, seed, kmax):
     np.testing.assert_array_equal(lens.cpu().numpy(), new_lens)
 
 
-def test_device_errors_are_flagged_not_fatal(S):
-    case = (4, 32, 8, 128, 4, 100, True, 1.0)
+@pytest.mark.parametrize("case", [(4, 32, 8, 128, 4, 100, True, 1.0),
+                                  (4, 16, 4, 64, 4, 100, True, 1.0)],
+                         ids=["query_rows_D128", "keys_as_rows_D64"])
+def test_device_errors_are_flagged_not_fatal(S, case):
     c = make(S, 6, case)
     kv = kv_for(S, c, c["lens"] + c["n_q"])
     B = case[0]
