@@ -134,6 +134,25 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, Ctrl* 
   return __all_sync(0xffffffffu, wait_or_abort(bar, parity, c, err));
 }
 
+// The softmax and epilogue warps' waits: try_wait without a sleep hint, so the
+// warp resumes as soon as the phase completes (a sleeping wait's wake-up
+// comes later, which each tile of a short launch pays in full); bounded like
+// wait_or_abort (the abort flag is read every 64 tries).
+__device__ __noinline__ bool wait_hot(uint64_t* bar, uint32_t parity, Ctrl* c, int32_t* err) {
+  for (uint32_t i = 0; i < (1u << 22); ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((i & 63u) == 63u && c->abort_flag) return false;
+  }
+  c->abort_flag = 1;
+  raise_err(err, SEED_DEVERR_TIMEOUT);
+  return false;
+}
+
+__device__ __forceinline__ bool warp_wait_hot(uint64_t* bar, uint32_t parity, Ctrl* c,
+                                              int32_t* err) {
+  return __all_sync(0xffffffffu, wait_hot(bar, parity, c, err));
+}
+
 // ------------------------------------------------------------- the kernel
 // One softmax row: the visible columns of a tile for query j are the cache
 // columns c <= lim (c < dcol) and the draft columns dcol <= c < dend.
@@ -713,7 +732,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
       const int s = t % kStagesTC;
       // S(t) done implies K(t) landed and tile t's descriptor is written; the
       // MMA thread also completes this phase, without an S, at the end
-      if (!warp_wait(&ctrl->s_full[par], own & 1, ctrl, p.err)) break;
+      if (!warp_wait_hot(&ctrl->s_full[par], own & 1, ctrl, p.err)) break;
       if (t >= *reinterpret_cast<volatile int32_t*>(&ctrl->end_tile)) break;
       const TileMeta m = ctrl->meta[t % kMetaRing];
       tc_fence_after();
@@ -765,7 +784,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
       // 0 never meets a stale or NaN-poisoned row
       if (m.cvalid - m.tile * kN < kN || cm.dcol < kN) {
         // (after V has landed, or the copy engine would overwrite the zeros)
-        if (!warp_wait(&ctrl->v_full[s], (t / kStagesTC) & 1, ctrl, p.err)) break;
+        if (!warp_wait_hot(&ctrl->v_full[s], (t / kStagesTC) & 1, ctrl, p.err)) break;
         uint8_t* vb = smem + kOffV + (size_t)s * kKV;
         bool wrote = false;
 #pragma unroll 1
@@ -784,12 +803,12 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
       // this group's previous PV must be done before its O is rescaled (the
       // rescale is rare: only when the running maximum jumps by > 2^8)
       const bool do_resc = warp_active && __any_sync(kFull, resc);
-      if (own > 0 && do_resc && !warp_wait(&ctrl->o_full[par], (own - 1) & 1, ctrl, p.err))
+      if (own > 0 && do_resc && !warp_wait_hot(&ctrl->o_full[par], (own - 1) & 1, ctrl, p.err))
         break;
       // the first tile of a unit overwrites O: the other group's epilogue of
       // the previous unit must have read it
       if (first_own && pend_rel) {
-        if (!warp_wait(&ctrl->orel_bar[q4], (xcnt - 1) & 1, ctrl, p.err)) break;
+        if (!warp_wait_hot(&ctrl->orel_bar[q4], (xcnt - 1) & 1, ctrl, p.err)) break;
         pend_rel = false;
       }
       tc_fence_after();
@@ -812,7 +831,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
 
       if (m.k + 2 >= m.ntu) {
         // ------------------------------------------------ this group's last tile of the unit
-        if (!warp_wait(&ctrl->o_full[par], own & 1, ctrl, p.err)) break;
+        if (!warp_wait_hot(&ctrl->o_full[par], own & 1, ctrl, p.err)) break;
         tc_fence_after();
         if (m.k != m.ntu - 1) {
           // the other group owns the epilogue: hand over this row's statistics
@@ -827,7 +846,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
           // ---------------------------------------------- epilogue (owner)
           float mo = -INFINITY, lo = 0.f;
           if (m.ntu >= 2) {
-            if (!warp_wait(&ctrl->stats_bar[q4], xcnt & 1, ctrl, p.err)) break;
+            if (!warp_wait_hot(&ctrl->stats_bar[q4], xcnt & 1, ctrl, p.err)) break;
             tc_fence_after();
             mo = ctrl->xm[q4][lane];
             lo = ctrl->xl[q4][lane];
