@@ -201,15 +201,12 @@ __device__ __noinline__ bool kt_poll1(uint64_t* bar, uint32_t parity, KtCtrl* c,
   return false;
 }
 
-// A whole warp waits on a hot barrier: lane 0 polls alone (one shared-memory
-// access per try instead of 32), then every lane acquires the phase.
+// A whole warp waits on a hot barrier, every lane polling (measured faster
+// than lane 0 polling alone and the others taking the phase after a
+// shuffle); the lanes agree on the outcome.
 __device__ __forceinline__ bool kt_warp_poll(uint64_t* bar, uint32_t parity, KtCtrl* c,
                                              int32_t* err) {
-  int ok = 0;
-  if ((threadIdx.x & 31) == 0) ok = kt_poll1(bar, parity, c, err) ? 1 : 0;
-  ok = __shfl_sync(kFull, ok, 0);
-  if (ok) mbar_test(bar, parity);
-  return ok != 0;
+  return __all_sync(kFull, kt_poll1(bar, parity, c, err));
 }
 
 // Exchange point of the eight softmax warps (an mbarrier counting one
