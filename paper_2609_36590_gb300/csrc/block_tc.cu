@@ -81,18 +81,9 @@ struct BlockTcParams {
   float c2;            // softmax scale * log2(e)
 };
 
-__device__ __noinline__ bool bwait(uint64_t* bar, uint32_t parity, BCtrl* c, int32_t* err) {
-  for (uint32_t i = 0; i < kSuspendTries; ++i) {
-    if (mbar_try_wait_sleep(bar, parity, kSuspendNs)) return true;
-    if (c->abort_flag) return false;
-  }
-  c->abort_flag = 1;
-  raise_err(err, SEED_DEVERR_TIMEOUT);
-  return false;
-}
-
-// A wait on the softmax warps' critical path: try_wait without a sleep hint
-// (the thread resumes as soon as the phase completes), bounded like bwait.
+// The softmax and epilogue warps' waits: try_wait without a sleep hint (the
+// thread resumes as soon as the phase completes; a sleeping wait wakes
+// later), bounded (2^22 tries; the abort flag is read every 64).
 __device__ __forceinline__ bool bwait_hot(uint64_t* bar, uint32_t parity, BCtrl* c, int32_t* err) {
   for (uint32_t i = 0; i < (1u << 22); ++i) {
     if (mbar_try_wait(bar, parity)) return true;
@@ -106,11 +97,6 @@ __device__ __forceinline__ bool bwait_hot(uint64_t* bar, uint32_t parity, BCtrl*
 __device__ __forceinline__ bool bwarp_hot(uint64_t* bar, uint32_t parity, BCtrl* c,
                                           int32_t* err) {
   return __all_sync(kBFull, bwait_hot(bar, parity, c, err));
-}
-
-__device__ __forceinline__ bool bwarp_wait(uint64_t* bar, uint32_t parity, BCtrl* c,
-                                           int32_t* err) {
-  return __all_sync(kBFull, bwait(bar, parity, c, err));
 }
 
 __device__ __forceinline__ bool bpoll(uint64_t* bar, uint32_t parity, BCtrl* c, int32_t* err) {
@@ -525,10 +511,10 @@ __global__ void __launch_bounds__(kBThreads, 1) block_tc_kernel(
       // piece; 16-byte chunks swizzled by row).
       if (pend && (t == 0 || !active)) {
         pend = false;
-        ok = bwarp_wait(&ctrl->l_full[pwi & 1], (uint32_t)((pwi >> 1) & 1), ctrl, p.err);
+        ok = bwarp_hot(&ctrl->l_full[pwi & 1], (uint32_t)((pwi >> 1) & 1), ctrl, p.err);
         if (!ok) break;
         const float el = ls_sh[(pwi & 1) * 256 + row] + ls_sh[(pwi & 1) * 256 + 128 + row];
-        ok = bwarp_wait(&ctrl->o_done[pwi & 1], (uint32_t)((pwi >> 1) & 1), ctrl, p.err);
+        ok = bwarp_hot(&ctrl->o_done[pwi & 1], (uint32_t)((pwi >> 1) & 1), ctrl, p.err);
         if (!ok) break;
         tc_fence_after();
         const uint32_t ocol = tmem + lane_off + kBColO + (uint32_t)(pwi & 1) * kBD + 64u * hf;
