@@ -516,8 +516,11 @@ __global__ void __launch_bounds__(kThreadsKT, 1)
           raise_err(p.err, SEED_DEVERR_PAGE);
           pid = -1;
         }
-        const int dslot = sq.nd > 0 ? sq.ncp - t * kPagesPerTile : -1;
-        const bool has = lane < kPagesPerTile && (pid >= 0 || lane == dslot);
+        // slot of draft page 0 (may lie outside the tile); lane pp holds
+        // draft page dpage when the tile's slot pp is one
+        const int dslot = sq.ncp - t * kPagesPerTile;
+        const int dpage = lane < kPagesPerTile ? draft_page_of_slot(sq.ncp, sq.nd, t, lane) : -1;
+        const bool has = lane < kPagesPerTile && (pid >= 0 || dpage >= 0);
         const uint32_t loads = __ballot_sync(kFull, has);
         const int box = box_size(pid, lane);
         KtMeta& m = ctrl->meta[mi];
@@ -552,10 +555,10 @@ __global__ void __launch_bounds__(kThreadsKT, 1)
         if (box > 0 || (has && pid < 0)) {
           uint8_t* kb = smem + LY.off_k + (size_t)s * GE::kTile + lane * 2048u;
           const CUtensorMap* mk = box > 0 ? &pm.k[log2_box(box)] : &tm_dk;
-          const int w = box > 0 ? pid : b;
+          const int w = box > 0 ? pid : b, r0 = box > 0 ? 0 : kPage * dpage;
 #pragma unroll
           for (int h = 0; h < GE::kSlabs; ++h)
-            tma_load_4d(kb + h * (kKeys * 128), mk, 64 * h, 0, g, w, &ctrl->k_full[s]);
+            tma_load_4d(kb + h * (kKeys * 128), mk, 64 * h, r0, g, w, &ctrl->k_full[s]);
         }
       }
       if (!ok) break;
@@ -593,13 +596,16 @@ __global__ void __launch_bounds__(kThreadsKT, 1)
       const KtMeta& m = ctrl->meta[mi];
       if (m.unit < 0) break;
       const int pid = lane < kPagesPerTile ? m.pids[lane] : -1;
-      const int mb = m.b, mg = m.g, dslot = m.dslot;
+      const int mb = m.b, mg = m.g, dslot = m.dslot, nd = m.nd;
       __syncwarp();
       if (lane == 0) mbar_arrive(&ctrl->meta_empty[mi]);
       if (tv >= GE::kSV &&
           !kt_warp_wait(&ctrl->v_empty[s], ((tv / GE::kSV) - 1) & 1, ctrl, p.err))
         break;
-      const bool has = lane < kPagesPerTile && (pid >= 0 || lane == dslot);
+      const int dpage =
+          (lane < kPagesPerTile && lane >= dslot && lane - dslot < draft_pages(nd)) ? lane - dslot
+                                                                                     : -1;
+      const bool has = lane < kPagesPerTile && (pid >= 0 || dpage >= 0);
       const uint32_t loads = __ballot_sync(kFull, has);
       if (lane == 0)
         mbar_arrive_expect_tx(&ctrl->v_full[s], (uint32_t)__popc(loads) * GE::kSlabs * 2048u);
@@ -608,10 +614,10 @@ __global__ void __launch_bounds__(kThreadsKT, 1)
       if (box > 0 || (has && pid < 0)) {
         uint8_t* vb = smem + LY.off_v + (size_t)s * GE::kTile + lane * 2048u;
         const CUtensorMap* mv = box > 0 ? &pm.v[log2_box(box)] : &tm_dv;
-        const int w = box > 0 ? pid : mb;
+        const int w = box > 0 ? pid : mb, r0 = box > 0 ? 0 : kPage * dpage;
 #pragma unroll
         for (int h = 0; h < GE::kSlabs; ++h)
-          tma_load_4d(vb + h * (kKeys * 128), mv, 64 * h, 0, mg, w, &ctrl->v_full[s]);
+          tma_load_4d(vb + h * (kKeys * 128), mv, 64 * h, r0, mg, w, &ctrl->v_full[s]);
       }
     }
     __syncwarp();

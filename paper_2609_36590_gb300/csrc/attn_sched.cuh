@@ -6,7 +6,8 @@
 // What a sequence sees (Sec. 4.1, Alg. 2): in draft mode one query over cache
 // rows 0 .. L - 1 followed by draft rows 0 .. nd - 1 of the draft scratch; in
 // verify mode query j < n_q over cache rows 0 .. L + j.  Rows are handled in
-// 16-token pages; 8 pages make a 128-row tile.
+// 16-token pages (the draft rows in one or two pages after the cache pages);
+// 8 pages make a 128-row tile.
 #pragma once
 
 #include <cuda.h>
@@ -28,6 +29,17 @@ struct SeqT {
   int nq, nd, ncp, cvalid, lim0, tiles, bad;
 };
 
+// Pages that hold nd draft rows: rows 16 i .. 16 i + 15 of the draft scratch
+// make draft page i, placed after the sequence's cache pages.
+__device__ __forceinline__ int draft_pages(int nd) { return (nd + kPage - 1) / kPage; }
+
+// Draft page held by page slot `slot` of tile t (-1: none), for a sequence
+// with ncp cache pages and nd draft rows.
+__device__ __forceinline__ int draft_page_of_slot(int ncp, int nd, int t, int slot) {
+  const int dp = t * kPagesPerTile + slot - ncp;
+  return (dp >= 0 && dp < draft_pages(nd)) ? dp : -1;
+}
+
 // Geometry of sequence b: query positions nq, draft rows nd, cache pages ncp,
 // rows that exist cvalid, query j sees cache positions <= lim0 + j, tiles.
 // A sequence with bad arguments (bad != 0) or no queries has no tiles.
@@ -45,7 +57,7 @@ __device__ __forceinline__ SeqT seq_of(const AttnTcParams& p, int b) {
     s.cvalid = L;
     s.lim0 = L - 1;
     s.ncp = (L + kPage - 1) / kPage;
-    s.tiles = (s.ncp + 1 + kPagesPerTile - 1) / kPagesPerTile;
+    s.tiles = (s.ncp + draft_pages(a) + kPagesPerTile - 1) / kPagesPerTile;
   } else {
     if (a < 0 || a > p.kmax + 1) s.bad |= SEED_DEVERR_NQ;
     if (L < 0 || (long long)L + a > cap) s.bad |= SEED_DEVERR_CTX_LEN;

@@ -91,7 +91,7 @@ struct TileMeta {
   int32_t cvalid;      // cache rows that exist (L, or L + n_q for verify)
   int32_t lim0;        // query j sees cache positions <= lim0 + j
   int32_t slot;        // partial record of this piece, or -1: the whole pair
-  int32_t dslot;       // page slot of the draft rows in this tile, or -1
+  int32_t dslot;       // page slot of draft page 0 (outside [0, 8) when not in this tile)
   int32_t pad[3];
   int32_t pids[kPagesPerTile];   // cache page of each page slot, -1: none
 };
@@ -516,8 +516,11 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
           pid = -1;
         }
         // lane pp < 8 owns page slot pp of the tile
-        const int dslot = sq.nd > 0 ? sq.ncp - t * kPagesPerTile : -1;
-        const bool has = lane < kPagesPerTile && (pid >= 0 || lane == dslot);
+        // slot of draft page 0 (may lie outside the tile); lane pp holds
+        // draft page dpage when the tile's slot pp is one
+        const int dslot = sq.ncp - t * kPagesPerTile;
+        const int dpage = lane < kPagesPerTile ? draft_page_of_slot(sq.ncp, sq.nd, t, lane) : -1;
+        const bool has = lane < kPagesPerTile && (pid >= 0 || dpage >= 0);
         const uint32_t loads = __ballot_sync(kFull, has);
         const int box = box_size(pid, lane);
         TileMeta& m = ctrl->meta[mi];
@@ -552,9 +555,9 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
           // a box of `box` pages from this slot on, or the draft rows' page
           uint8_t* kb = smem + kOffK + (size_t)s * kKV + lane * 2048u;
           const CUtensorMap* mk = box > 0 ? &pm.k[log2_box(box)] : &tm_dk;
-          const int w = box > 0 ? pid : b;
-          tma_load_4d(kb, mk, 0, 0, g, w, &ctrl->k_full[s]);
-          tma_load_4d(kb + kHalf, mk, 64, 0, g, w, &ctrl->k_full[s]);
+          const int w = box > 0 ? pid : b, r0 = box > 0 ? 0 : kPage * dpage;
+          tma_load_4d(kb, mk, 0, r0, g, w, &ctrl->k_full[s]);
+          tma_load_4d(kb + kHalf, mk, 64, r0, g, w, &ctrl->k_full[s]);
         }
       }
       if (!ok) break;
@@ -593,13 +596,16 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
       const TileMeta& m = ctrl->meta[mi];
       if (m.unit < 0) break;
       const int pid = lane < kPagesPerTile ? m.pids[lane] : -1;
-      const int mb = m.b, mg = m.g, dslot = m.dslot;
+      const int mb = m.b, mg = m.g, dslot = m.dslot, nd = m.nd;
       __syncwarp();
       if (lane == 0) mbar_arrive(&ctrl->meta_empty[mi]);
       if (tv >= kStagesTC &&
           !warp_wait(&ctrl->v_empty[s], ((tv / kStagesTC) - 1) & 1, ctrl, p.err))
         break;
-      const bool has = lane < kPagesPerTile && (pid >= 0 || lane == dslot);
+      const int dpage =
+          (lane < kPagesPerTile && lane >= dslot && lane - dslot < draft_pages(nd)) ? lane - dslot
+                                                                                     : -1;
+      const bool has = lane < kPagesPerTile && (pid >= 0 || dpage >= 0);
       const uint32_t loads = __ballot_sync(kFull, has);
       if (lane == 0)
         mbar_arrive_expect_tx(&ctrl->v_full[s], (uint32_t)__popc(loads) * 2u * 2048u);
@@ -608,9 +614,9 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
       if (box > 0 || (has && pid < 0)) {
         uint8_t* vb = smem + kOffV + (size_t)s * kKV + lane * 2048u;
         const CUtensorMap* mv = box > 0 ? &pm.v[log2_box(box)] : &tm_dv;
-        const int w = box > 0 ? pid : mb;
-        tma_load_4d(vb, mv, 0, 0, mg, w, &ctrl->v_full[s]);
-        tma_load_4d(vb + kHalf, mv, 64, 0, mg, w, &ctrl->v_full[s]);
+        const int w = box > 0 ? pid : mb, r0 = box > 0 ? 0 : kPage * dpage;
+        tma_load_4d(vb, mv, 0, r0, mg, w, &ctrl->v_full[s]);
+        tma_load_4d(vb + kHalf, mv, 64, r0, mg, w, &ctrl->v_full[s]);
       }
     }
     __syncwarp();

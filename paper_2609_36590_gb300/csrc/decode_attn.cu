@@ -73,7 +73,8 @@ __device__ __forceinline__ Seq load_seq(const DecodeParams& p, int v) {
     s.nctx = L;
     s.ndraft = dl;
   }
-  s.npages = (s.nctx + kPage - 1) / kPage + (s.ndraft > 0 ? 1 : 0);
+  // the draft rows fill one or two pages after the cache pages
+  s.npages = (s.nctx + kPage - 1) / kPage + (s.ndraft + kPage - 1) / kPage;
   return s;
 }
 
@@ -127,7 +128,7 @@ __device__ __forceinline__ int page_rows(const DecodeParams& p, const Seq& s, in
     return min(kPage, s.nctx - pg * kPage);
   }
   *pid_out = -1;
-  return s.ndraft;
+  return min(kPage, s.ndraft - (pg - ctx_pages(s)) * kPage);   // draft page pg - ctx_pages
 }
 
 // Producer: one thread puts the K and V pages of the cursor's current tile
@@ -157,7 +158,8 @@ __device__ void issue_tile(const DecodeParams& p, const Cursor& cu, int stage, u
       src_v[w] = p.v_cache + off;
       bytes[w] = kPage * D * 2;   // whole page; rows past the length are masked
     } else {
-      const size_t off = ((size_t)cu.s.b * p.hkv + cu.g) * p.kmax * D;
+      const size_t off =
+          (((size_t)cu.s.b * p.hkv + cu.g) * p.kmax + (size_t)(pg - ctx_pages(cu.s)) * kPage) * D;
       src_k[w] = p.draft_k + off;
       src_v[w] = p.draft_v + off;
       bytes[w] = (uint32_t)rows * D * 2;
@@ -469,7 +471,7 @@ DecodePlan plan_decode(int32_t nv, int32_t hkv, int32_t group, int32_t head_dim,
                        int32_t max_pages) {
   DecodePlan pl{};
   pl.nv = nv;
-  const long long pages_cap = (long long)max_pages + 1;
+  const long long pages_cap = (long long)max_pages + 2;   // + up to two draft pages
   const long long total = (long long)nv * hkv * pages_cap;
   long long ppu = 4 * ((total + 4LL * kTargetUnits - 1) / (4LL * kTargetUnits));
   if (ppu < 4) ppu = 4;

@@ -68,6 +68,13 @@ CASES = [
     # many CTAs, G = 8 query heads per KV head
     (9, 8, 1, 128, 4, 3000, True, 1.0),
     (16, 8, 1, 128, 8, 1100, True, 1.0),
+    # more than 16 draft rows: the draft rows span two pages (one of them
+    # may open the next 128-row tile)
+    (6, 32, 8, 128, 24, 300, True, 1.0),
+    (4, 8, 8, 128, 31, 150, True, 1.0),
+    (6, 16, 8, 64, 20, 200, True, 1.0),
+    # head_dim 64 with 72 query rows per KV head: the CUDA-core verify route
+    (4, 64, 8, 64, 8, 300, True, 1.0),
 ]
 
 
@@ -121,6 +128,28 @@ def test_draft_attention_matches_oracle(S, case):
         if dl == 0:
             assert (out[b] == SENTINEL).all() and (lse[b] == SENTINEL).all()
             continue
+        o, l = OAT.draft_attention_seq(
+            f64(c["q_draft"][b]), f64(c["rows_k"][b, :L]), f64(c["rows_v"][b, :L]),
+            f64(c["draft_k"][b, :, :dl].transpose(1, 0, 2)),
+            f64(c["draft_v"][b, :, :dl].transpose(1, 0, 2)), c["scale"])
+        assert_close(out[b], o, f"draft o b={b} L={L} dl={dl}")
+        assert_close(lse[b], l, f"draft lse b={b}")
+
+
+@pytest.mark.parametrize("case", [(8, 32, 8, 128, 24, 260, True, 1.0),
+                                  (8, 16, 8, 64, 20, 260, True, 1.0)],
+                         ids=["D128_G4", "D64_G2"])
+def test_draft_rows_span_pages_and_tiles(S, case):
+    """More than 16 draft rows fill two pages after the cache pages; with 7 or
+    15 cache pages the second draft page opens the next 128-row tile."""
+    c = make(S, 3, case)
+    kmax = case[4]
+    c["lens"] = np.array([97, 112, 111, 240, 225, 0, 16, 255], dtype=np.int32)
+    c["draft_lens"] = np.minimum(np.array([17, 24, 16, 20, 24, 18, 23, 1]), kmax).astype(np.int32)
+    out, lse = run_draft(S, c, kv_for(S, c, c["lens"]))
+    assert int(c["err"].item()) == 0
+    for b in range(case[0]):
+        dl, L = int(c["draft_lens"][b]), int(c["lens"][b])
         o, l = OAT.draft_attention_seq(
             f64(c["q_draft"][b]), f64(c["rows_k"][b, :L]), f64(c["rows_v"][b, :L]),
             f64(c["draft_k"][b, :, :dl].transpose(1, 0, 2)),
