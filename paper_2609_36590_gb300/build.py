@@ -20,7 +20,7 @@ BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libseed.so")
 
 SOURCES = ["seed_api.cu", "decode_attn.cu", "cache_accept.cu", "attn_tc.cu", "attn_kt.cu",
-           "noalloc_api.cu",
+           "attn_cluster.cu", "noalloc_api.cu",
            "head_tc.cu", "linear_tc.cu", "draft_ops.cu", "draft_api.cu",
            "block_attn.cu", "block_tc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]

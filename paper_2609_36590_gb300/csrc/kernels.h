@@ -206,4 +206,17 @@ cudaError_t launch_attn_kt(const AttnTcParams& p, int head_dim, const void* q,
                            const void* k_cache, const void* v_cache, const void* draft_k,
                            const void* draft_v, cudaStream_t st);
 
+// Cluster attention for launches with few (sequence, KV head) pairs
+// (attn_cluster.cu): one cluster of 8, 12 or 16 CTAs per pair, each CTA at
+// most kClMaxPages pages of the pair, at most kClRows query rows per KV head,
+// head_dim 128.  attn_cl_route gives the cluster size for a launch (0: not
+// this kernel): the largest whose clusters are all resident at once and whose
+// CTAs hold every sequence the page table allows.
+constexpr int kClMaxPages = 19;
+constexpr int kClRows = 32;
+int attn_cl_route(int head_dim, int group, int w1, int batch, int hkv, int max_pages);
+cudaError_t launch_attn_cl(const AttnTcParams& p, int cluster, const void* k_cache,
+                           const void* v_cache, const void* draft_k, const void* draft_v,
+                           cudaStream_t st);
+
 }  // namespace seedk

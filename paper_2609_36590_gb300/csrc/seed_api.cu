@@ -103,9 +103,11 @@ seed_status_t run_decode(const seed_cfg_t* cfg, int32_t batch, bool verify, cons
   return finish(seedk::launch_decode(p, cfg->head_dim, G, static_cast<cudaStream_t>(stream)));
 }
 
-// Draft / verify attention on the tensor cores: the keys-as-rows kernel for
-// head_dim 64 when the R = G * W1 query rows of a KV head fit 48 MMA
-// columns, the query-rows kernel for head_dim 128 (R <= 128).
+// Draft / verify attention on the tensor cores: the cluster kernel when the
+// launch has few (sequence, KV head) pairs and short sequences (head_dim 128,
+// R = G * W1 <= 32), else the keys-as-rows kernel for head_dim 64 when the R
+// query rows of a KV head fit 48 MMA columns, the query-rows kernel for
+// head_dim 128 (R <= 128).
 seed_status_t run_attn_tc(const seed_cfg_t* cfg, int32_t batch, bool draft, const void* q,
                           const int32_t* aux, const seed_kv_t& kv, const void* draft_k,
                           const void* draft_v, const int32_t* ctx_lens, float* out, float* lse,
@@ -147,6 +149,11 @@ seed_status_t run_attn_tc(const seed_cfg_t* cfg, int32_t batch, bool draft, cons
   p.draft_v = static_cast<const uint16_t*>(draft_v);
   p.D = cfg->head_dim;
   const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const int cluster =
+      anc == nullptr ? seedk::attn_cl_route(cfg->head_dim, G, W1, batch, cfg->hkv, kv.max_pages)
+                     : 0;
+  if (cluster > 0)
+    return finish(seedk::launch_attn_cl(p, cluster, kv.k, kv.v, draft_k, draft_v, st));
   return finish(kt ? seedk::launch_attn_kt(p, cfg->head_dim, q, kv.k, kv.v, draft_k, draft_v, st)
                    : seedk::launch_attn_tc(p, q, kv.k, kv.v, draft_k, draft_v, st));
 }

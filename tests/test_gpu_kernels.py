@@ -75,6 +75,14 @@ CASES = [
     (6, 16, 8, 64, 20, 200, True, 1.0),
     # head_dim 64 with 72 query rows per KV head: the CUDA-core verify route
     (4, 64, 8, 64, 8, 300, True, 1.0),
+    # few pairs, short page tables, <= 32 query rows: the cluster kernel
+    # (clusters of 16, 12 or 8 CTAs for up to 7, 8 and 15 pairs on a
+    # GB300), with 8, 16, 24 and 32 query rows, two draft pages and x8 keys
+    (8, 4, 1, 128, 7, 2000, True, 1.0),
+    (2, 16, 2, 128, 3, 900, True, 8.0),
+    (3, 8, 4, 128, 7, 1500, False, 1.0),
+    (2, 4, 4, 128, 24, 400, True, 1.0),
+    (5, 8, 2, 128, 4, 2300, True, 1.0),
 ]
 
 
@@ -174,6 +182,38 @@ def test_verify_attention_matches_oracle(S, case):
         assert_close(lse[b, :n], l, f"verify lse b={b}")
 
 
+@pytest.mark.parametrize("nq,dl", [((5, 3, 2), (4, 1, 2)), ((1, 5, 4), (2, 4, 3))])
+def test_few_pairs_at_the_page_limit(S, nq, dl):
+    """Three sequences x four KV heads (12 pairs, G = 4, k = 4): the cluster
+    kernel with clusters of 8 CTAs, one sequence of 149 cache pages (the
+    CTAs of its pairs at their 19-page limit), one near 2048 tokens."""
+    case = (3, 16, 4, 128, 4, 2370, True, 1.0)
+    c = make(S, 4, case)
+    assert c["max_pages"] + 2 <= 8 * 19
+    c["lens"] = np.array([2370, 2047, 100], dtype=np.int32)
+    c["n_q"] = np.array(nq, dtype=np.int32)
+    c["draft_lens"] = np.array(dl, dtype=np.int32)
+    out, lse = run_verify(S, c, kv_for(S, c, c["lens"] + c["n_q"]))
+    assert int(c["err"].item()) == 0
+    for b in range(3):
+        n, L = int(c["n_q"][b]), int(c["lens"][b])
+        assert (out[b, n:] == SENTINEL).all()
+        o, l = OAT.verify_attention_seq(f64(c["q_verify"][b, :n]), f64(c["rows_k"][b, :L + n]),
+                                        f64(c["rows_v"][b, :L + n]), L, c["scale"])
+        assert_close(out[b, :n], o, f"verify o b={b} L={L} n={n}")
+        assert_close(lse[b, :n], l, f"verify lse b={b}")
+    out, lse = run_draft(S, c, kv_for(S, c, c["lens"]))
+    assert int(c["err"].item()) == 0
+    for b in range(3):
+        d, L = int(c["draft_lens"][b]), int(c["lens"][b])
+        o, l = OAT.draft_attention_seq(
+            f64(c["q_draft"][b]), f64(c["rows_k"][b, :L]), f64(c["rows_v"][b, :L]),
+            f64(c["draft_k"][b, :, :d].transpose(1, 0, 2)),
+            f64(c["draft_v"][b, :, :d].transpose(1, 0, 2)), c["scale"])
+        assert_close(out[b], o, f"draft o b={b} L={L} dl={d}")
+        assert_close(lse[b], l, f"draft lse b={b}")
+
+
 def spike_rows(c, which, step, log2_gap):
     """Key rows that score log2_gap (in log2 units of the softmax) above a
     typical score for query head G g of KV head g: every step-th visible row
@@ -196,8 +236,9 @@ def spike_rows(c, which, step, log2_gap):
 
 
 @pytest.mark.parametrize("case", [(10, 32, 8, 128, 4, 1100, True, 1.0),
-                                  (10, 16, 8, 64, 2, 900, True, 1.0)],
-                         ids=["D128_G4", "D64_G2"])
+                                  (10, 16, 8, 64, 2, 900, True, 1.0),
+                                  (8, 4, 1, 128, 4, 1100, True, 1.0)],
+                         ids=["D128_G4", "D64_G2", "D128_G4_few_pairs"])
 @pytest.mark.parametrize("gap", [40.0, 300.0], ids=["gap40", "gap300"])
 def test_late_score_spikes_match_oracle(S, case, gap):
     """Scores far above the first tile's maximum, in later tiles and in the
