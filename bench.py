@@ -101,6 +101,7 @@ KERNEL_SOURCES = {
     "attn_tc_kernel": ["attn_tc.cu", "attn_sched.cuh", "tc.cuh", "common.cuh", "kernels.h"],
     "attn_kt_kernel": ["attn_kt.cu", "attn_sched.cuh", "tc.cuh", "common.cuh", "kernels.h"],
     "decode_attn_kernel": ["decode_attn.cu", "common.cuh", "kernels.h"],
+    "attn_cl_kernel": ["attn_cluster.cu", "attn_sched.cuh", "tc.cuh", "common.cuh", "kernels.h"],
 }
 
 
@@ -440,10 +441,24 @@ def attn_call_bytes(wl, kind, key, lens, k_b) -> int:
 
 
 def attn_kernel_name(wl, kind: str = "verify") -> str:
-    """The kernel behind seed_draft_attn / seed_verify_attn for this shape:
-    head_dim 128 with the query rows of one KV head in one 128-row tile: the
-    query-rows tensor-core kernel; head_dim 64 with at most 48 such rows: the
-    keys-as-rows tensor-core kernel; else the CUDA-core split-KV kernel."""
+    """The kernel behind seed_draft_attn / seed_verify_attn ("draft",
+    "verify") or seed_tree_verify_attn ("tree") for this workload.  On a GPU
+    the library says (seed_attn_route: few (sequence, KV head) pairs and short
+    page tables take the cluster kernel); the shape rule below is the rest of
+    the choice: head_dim 128 with the query rows of one KV head in one 128-row
+    tile: the query-rows tensor-core kernel; head_dim 64 with at most 48 such
+    rows: the keys-as-rows tensor-core kernel; else the CUDA-core split-KV
+    kernel."""
+    if kind != "tree":
+        try:
+            import torch
+            if torch.cuda.is_available():
+                import paper_2609_36590_gb300 as seed
+                cfg = seed.SeedConfig(hq=wl.hq, hkv=wl.hkv, head_dim=wl.head_dim, kmax=wl.kmax)
+                r = seed.seed_attn_route(cfg, wl.batch, kind == "draft", gen.max_pages(wl))
+                return seed.ROUTE_KERNELS[r]
+        except (ImportError, OSError, RuntimeError):
+            pass
     G = wl.hq // wl.hkv
     w1 = 1 if kind == "draft" else wl.kmax + 1
     if wl.head_dim == 128 and G * w1 <= 128:
@@ -533,7 +548,7 @@ def run_profile(args):
     assert int(dw.err.item()) == 0, f"device error flag {int(dw.err.item())} raised"
     key = (1, dec[0]) if args.profile == "draft" else dec[0]
     nbytes = attn_call_bytes(wl, "draft" if args.profile == "draft" else "verify", key, lens, k_b)
-    kname = attn_kernel_name(wl, "draft" if args.profile == "draft" else "verify")
+    kname = attn_kernel_name(wl, args.profile)
     print(json.dumps({"profile": args.profile, "workload": wl.name,
                       "kernel": kname, "sources": kernel_source_hash(kname),
                       "alg_bytes_per_launch": nbytes,

@@ -45,7 +45,7 @@
 extern "C" {
 #endif
 
-#define SEED_ABI_VERSION 3
+#define SEED_ABI_VERSION 4
 #define SEED_MAX_KMAX 31        /* largest supported draft length d (32 rows per sequence) */
 
 typedef enum {
@@ -168,6 +168,32 @@ seed_status_t seed_verify_attn(const seed_cfg_t* cfg, int32_t batch, const void*
                                const int32_t* n_q, seed_kv_t kv, const int32_t* ctx_lens,
                                float* out, float* lse, void* ws, size_t ws_bytes,
                                int32_t* err_flag, void* stream);
+
+/* Which kernel seed_draft_attn (draft != 0) or seed_verify_attn (draft == 0)
+ * runs for this cfg, batch and page-table width max_pages on the current
+ * device (the calls choose the same way; for diagnostics and tests):
+ *   SEED_ROUTE_CUDA_CORE   split-KV kernel on CUDA cores
+ *   SEED_ROUTE_TC_ROWS     tensor cores, the query rows of a KV head as MMA
+ *                          rows (head_dim 128, up to 128 rows)
+ *   SEED_ROUTE_TC_KEYS     tensor cores, the keys as MMA rows (head_dim 64,
+ *                          up to 48 query rows)
+ *   SEED_ROUTE_CLUSTER_8, _12, _16
+ *                          few (sequence, KV head) pairs and short page tables
+ *                          (head_dim 128, up to 32 query rows): one cluster of
+ *                          8, 12 or 16 CTAs per pair, merged on chip; the
+ *                          largest cluster whose clusters all fit the device
+ *                          at once and whose CTAs hold max_pages + 2 pages
+ * seed_tree_verify_attn always takes a tensor-core route.  Returns -1 for an
+ * invalid cfg, batch < 1 or max_pages < 1. */
+typedef enum {
+  SEED_ROUTE_CUDA_CORE = 0,
+  SEED_ROUTE_TC_ROWS = 1,
+  SEED_ROUTE_TC_KEYS = 2,
+  SEED_ROUTE_CLUSTER_8 = 8,
+  SEED_ROUTE_CLUSTER_12 = 12,
+  SEED_ROUTE_CLUSTER_16 = 16
+} seed_route_t;
+int32_t seed_attn_route(const seed_cfg_t* cfg, int32_t batch, int32_t draft, int32_t max_pages);
 
 /* Greedy acceptance and cache commit/rollback (Alg. 2, after verification):
  * n_b = number of leading i < k_b[b] with draft_ids[b,i] == target_ids[b,i];

@@ -58,6 +58,7 @@ _SIGS = {
     "seed_abi_version": (_I, []),
     "seed_status_string": (ctypes.c_char_p, [_I]),
     "seed_workspace_bytes": (ctypes.c_size_t, [ctypes.POINTER(_Cfg), _I]),
+    "seed_attn_route": (_I, [ctypes.POINTER(_Cfg), _I, _I, _I]),
     "seed_draft_kv_append": (_I, [ctypes.POINTER(_Cfg), _I, _P, _P, _P, _P, _P, _P, _P]),
     "seed_draft_attn": (_I, [ctypes.POINTER(_Cfg), _I, _P, _KV, _P, _P, _P, _P, _P, _P, _P,
                              ctypes.c_size_t, _P, _P]),
@@ -188,6 +189,20 @@ def seed_workspace_bytes(cfg: SeedConfig, batch: int) -> int:
     if n == 0:
         raise SeedError("invalid configuration")
     return int(n)
+
+
+ROUTE_CUDA_CORE, ROUTE_TC_ROWS, ROUTE_TC_KEYS = 0, 1, 2
+ROUTE_KERNELS = {0: "decode_attn_kernel", 1: "attn_tc_kernel", 2: "attn_kt_kernel",
+                 8: "attn_cl_kernel", 12: "attn_cl_kernel", 16: "attn_cl_kernel"}
+
+
+def seed_attn_route(cfg: SeedConfig, batch: int, draft: bool, max_pages: int) -> int:
+    """The kernel seed_draft_attn (draft) or seed_verify_attn runs for this
+    shape on the current device: ROUTE_* or a cluster size 8, 12, 16."""
+    r = _lib.seed_attn_route(ctypes.byref(cfg.c()), batch, 1 if draft else 0, max_pages)
+    if r < 0:
+        raise SeedError(f"seed_attn_route: invalid arguments ({r})")
+    return r
 
 
 def new_workspace(cfg: SeedConfig, batch: int, device=None) -> torch.Tensor:

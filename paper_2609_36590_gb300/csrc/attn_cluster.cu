@@ -24,18 +24,20 @@
 //    verify pass) the copies start one load latency after the wait;
 //  * all of a CTA's pages (at most 19) land at once: one TMA copy per 64-dim
 //    half and run of consecutive page ids (1, 2, 4 or 8 pages; the copy
-//    engine takes ~30 ns per copy, so one copy per page would cost more than
-//    the data), one mbarrier per 128-key tile, and nothing waits for the copy
-//    warp but the products that need its pages;
+//    engine takes ~30 ns per copy), K of every tile before any V, one
+//    mbarrier per tile and tensor, and nothing waits for the copy warp but
+//    the products that need its pages;
 //  * products on the tensor cores with the keys as MMA rows:
 //      S^T = K Q^T   (tcgen05, M = 128 keys, N = 16 or 32 query rows),
 //      O^T = V^T P^T (M = 128 head dims, N = 64: P_hi and P_lo of 32 query
 //                    rows side by side, K = 16 keys per instruction);
 //    each 128-key tile has its own group of four softmax warps (one thread
-//    per key), its own maxima and its own O^T accumulator, so no tile waits
-//    for another's softmax; a thread reduces its query columns across the
-//    warp with a transposing butterfly (31 shuffles for 32 columns), and the
-//    epilogue adds the tiles' accumulators with weights 2^(m_t - M);
+//    per key), its own maxima and its own O^T accumulators, so no tile waits
+//    for another's softmax; only the NC query rows rounded up to 8 are read
+//    and exponentiated (8 for a draft call at G = 4), the column maxima and
+//    sums over a warp's 32 keys come from redux.sync (the sums on P in 24-bit
+//    fixed point), and the epilogue adds the tiles' accumulators with
+//    weights 2^(m_t - M);
 //  * each CTA sends its partial state to the CTA that owns each 1/S of the
 //    head dims with asynchronous distributed-shared-memory stores that count
 //    their bytes on the owner's mbarrier; an owner merges as soon as every
@@ -70,8 +72,10 @@ constexpr int kWarpMmaCl = 12, kWarpLoadCl = 13;   // MMA, copies and TMEM; Q
 constexpr int kClTiles = (kClMaxPages * kPage + 127) / 128;   // 128-key tiles: 3
 constexpr int kClKeys = kClMaxPages * kPage;                  // 304
 constexpr uint32_t kClTmemCols = 512;
-// TMEM columns: S^T of tile m at [32 m, 32 m + 32); O^T of tile m at
-// [128 + 64 m, 128 + 64 m + 64): P_hi columns, then P_lo columns
+// TMEM columns: S^T of tile m at [32 m, 32 m + 32); O^T of tile m in two
+// accumulators (even and odd pages, which halves the dependent chain of
+// products) at [128 + 128 m, + 64) and [192 + 128 m, + 64), each P_hi
+// columns then P_lo columns
 constexpr uint32_t kClColO = 128;
 constexpr float kClLn2 = 0.69314718055994531f;
 constexpr int kClRecvStride = 36;          // floats per received (source, dim) row of 32 columns
@@ -205,46 +209,66 @@ __device__ __forceinline__ bool cl_wait_cluster(uint64_t* bar, uint32_t parity) 
   return false;
 }
 
-// 32 consecutive TMEM columns of this thread's lane, or 16.
-template <int NQ>
-__device__ __forceinline__ void tmem_ld_cols(uint32_t taddr, float (&v)[NQ]) {
-  if constexpr (NQ == 32) {
+// N (8, 16, 24 or 32) consecutive TMEM columns of this thread's lane, added
+// to v (the loads are issued together and waited for once).
+template <int N>
+__device__ __forceinline__ void tmem_add_cols(uint32_t taddr, float (&v)[N]) {
+  static_assert(N % 8 == 0 && N <= 32, "column count");
+  if constexpr (N == 32) {
     uint32_t r[32];
     tmem_ld32(taddr, r);
     tmem_wait_ld();
 #pragma unroll
-    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
-  } else {
+    for (int i = 0; i < 32; ++i) v[i] += __uint_as_float(r[i]);
+  } else if constexpr (N == 24) {
+    uint32_t r[16], r2[8];
+    tmem_ld16(taddr, r);
+    tmem_ld8(taddr + 16, r2);
+    tmem_wait_ld();
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] += __uint_as_float(r[i]);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[16 + i] += __uint_as_float(r2[i]);
+  } else if constexpr (N == 16) {
     uint32_t r[16];
     tmem_ld16(taddr, r);
     tmem_wait_ld();
 #pragma unroll
-    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+    for (int i = 0; i < 16; ++i) v[i] += __uint_as_float(r[i]);
+  } else {
+    uint32_t r[8];
+    tmem_ld8(taddr, r);
+    tmem_wait_ld();
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[i] += __uint_as_float(r[i]);
   }
 }
 
-// Column reduction of a warp's 32 x NQ values (lane = row): a transposing
-// butterfly -- at each step a lane keeps half of its columns and takes its
-// partner's values for them -- leaves the result for column lane % NQ in
-// v[0] (NQ - 1 shuffles, plus one for NQ = 16).
-template <int NQ, bool MAX>
-__device__ __forceinline__ float col_reduce(float (&v)[NQ], int lane) {
-#pragma unroll
-  for (int off = NQ / 2; off >= 1; off >>= 1) {
-    const bool up = (lane & off) != 0;
-#pragma unroll
-    for (int i = 0; i < off; ++i) {
-      const float send = up ? v[i] : v[i + off];
-      const float keep = up ? v[i + off] : v[i];
-      const float r = __shfl_xor_sync(kFull, send, off);
-      v[i] = MAX ? fmaxf(keep, r) : keep + r;
-    }
+// Warp-wide sum of one value per lane (every lane gets it).
+__device__ __forceinline__ uint32_t warp_sum_u32(uint32_t x) {
+  uint32_t r;
+  asm volatile("redux.sync.add.u32 %0, %1, 0xffffffff;" : "=r"(r) : "r"(x));
+  return r;
+}
+
+// Warp-wide maximum of one value per lane (every lane gets it).
+__device__ __forceinline__ float warp_max(float x) {
+  float r;
+  asm volatile("redux.sync.max.f32 %0, %1, 0xffffffff;" : "=f"(r) : "f"(x));
+  return r;
+}
+
+// A tile's O^T columns 0 .. N - 1 of this thread's lane: the sum of its two
+// accumulators (even and odd pages; the odd one is unwritten when the tile
+// has a single page), each P_hi columns plus P_lo columns.
+template <int N>
+__device__ __forceinline__ void tile_o(uint32_t taddr, int pages, float (&o)[N]) {
+  tmem_add_cols<N>(taddr, o);
+  tmem_add_cols<N>(taddr + 32u, o);
+  if (pages >= 2) {
+    tmem_add_cols<N>(taddr + 64u, o);
+    tmem_add_cols<N>(taddr + 96u, o);
   }
-  if constexpr (NQ == 16) {
-    const float r = __shfl_xor_sync(kFull, v[0], 16);
-    v[0] = MAX ? fmaxf(v[0], r) : v[0] + r;
-  }
-  return v[0];
 }
 
 // Pages [p0, p0 + npg) of the np pages of a pair, for CTA `rank` of S.
@@ -294,13 +318,14 @@ __device__ __forceinline__ void prepare(const AttnTcParams& p, int b, int g, int
 
 // ------------------------------------------------------------- the kernel
 // Grid (S, hkv, B), clusters of S along x: cluster (b, g), CTA rank r.
-// NQ = query rows padded to the S MMA's N (16 or 32; G * W1 <= NQ).
-template <int D, int NQ, int S>
+// NC = query rows G * W1 rounded up to 8: the columns the softmax reads.
+template <int D, int NC, int S>
 __global__ void __launch_bounds__(kClThreads, 1)
     attn_cl_kernel(const __grid_constant__ PageMaps pm, const __grid_constant__ CUtensorMap tm_dk,
                    const __grid_constant__ CUtensorMap tm_dv, const AttnTcParams p) {
   using LY = ClLayout<D, S>;
   static_assert(D == 128, "the epilogue warps hold one head dim per thread");
+  constexpr int NQ = NC <= 16 ? 16 : 32;        // the S MMA's N
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   // 128-byte swizzled operands need a 1 KiB aligned base (the same offset in
   // every CTA, so the receive buffers sit at the same address in each)
@@ -510,7 +535,8 @@ __global__ void __launch_bounds__(kClThreads, 1)
         for (int kk = 8 * m; kk < k1; ++kk) {
           const uint64_t a = smem_desc_sw128(sV + kk * 2048u, LY::kHalfBytes, 1024);
           const uint64_t bp = smem_desc_sw128(sP + kk * 2048u, 0, 1024);
-          mma_ss(tmem + kClColO + 64u * m, a, bp, kIdescPV, kk > 8 * m);
+          const uint32_t acc = kClColO + 128u * m + 64u * ((kk - 8 * m) & 1);
+          mma_ss(tmem + acc, a, bp, kIdescPV, kk - 8 * m >= 2);
         }
         mma_commit(&ctrl->o_full[m]);
       }
@@ -531,83 +557,82 @@ __global__ void __launch_bounds__(kClThreads, 1)
       // keys past the CTA's pages (the end of the last tile) are never read
       // by PV and have no row in the P operand
       const bool in_pages = s < npg;
-      int nmin = NQ;   // first query row that sees the key (NQ: none)
+      int nmin = NC;   // first query row that sees the key (NC: none)
       const bool gotc = cl_warp_wait(&ctrl->codes_ready, 0);
       ok = ok && gotc;
       if (in_pages && gotc) {
         const int code = ctrl->code[s];
         if (code <= -2) {
-          nmin = (kPage * (-2 - code) + (key & 15) < sq.nd) ? 0 : NQ;
+          nmin = (kPage * (-2 - code) + (key & 15) < sq.nd) ? 0 : NC;
         } else if (code >= 0) {
           const int kpos = (p0 + s) * kPage + (key & 15);
-          nmin = kpos < sq.cvalid ? min(max(kpos - sq.lim0, 0) << lg, NQ) : NQ;
+          nmin = kpos < sq.cvalid ? min(max(kpos - sq.lim0, 0) << lg, NC) : NC;
         }
       }
       const bool got = cl_warp_wait(&ctrl->s_full[m], 0);
       ok = ok && got;
       tc_fence_after();
-      float v[NQ], sv[NQ];
-      if (got) {
-        tmem_ld_cols<NQ>(tmem + lane_off + 32u * m, v);
-      } else {
+      float sv[NC];
 #pragma unroll
-        for (int c = 0; c < NQ; ++c) v[c] = 0.f;
-      }
+      for (int c = 0; c < NC; ++c) sv[c] = 0.f;
+      if (got) tmem_add_cols<NC>(tmem + lane_off + 32u * m, sv);
 #pragma unroll
-      for (int c = 0; c < NQ; ++c) {
-        sv[c] = c >= nmin ? v[c] * c2 : -INFINITY;
-        v[c] = sv[c];
+      for (int c = 0; c < NC; ++c) sv[c] = c >= nmin ? sv[c] * c2 : -INFINITY;
+      // the tile's column maxima: over the warp's 32 keys, then the group's
+#pragma unroll
+      for (int c = 0; c < NC; ++c) {
+        const float wm = warp_max(sv[c]);
+        if (lane == 0) ctrl->wmax[m][q4][c] = wm;
       }
-      const float mx = col_reduce<NQ, true>(v, lane);
-      if (lane < NQ) ctrl->wmax[m][q4][lane] = mx;
       tile_bar(m);
-      if (q4 == 0 && lane < NQ) {
+      if (q4 == 0 && lane < NC) {
         float t = -INFINITY;
 #pragma unroll
         for (int w = 0; w < 4; ++w) t = fmaxf(t, ctrl->wmax[m][w][lane]);
         ctrl->tmax[m][lane] = t;
       }
       tile_bar(m);
-      // P^T row of this key: P_hi of query rows 0-31 (chunks 0-3), then P_lo
-      // (chunks 4-7); rows past NQ are zero
-      uint32_t hi[16], lo[16];
+      // P^T row of this key: P_hi of query rows 0-31 (16-byte chunks 0-3),
+      // then P_lo (chunks 4-7); only the chunks of the NC rows are written
+      // (the others feed output columns nobody reads)
+      float pv[NC];
 #pragma unroll
-      for (int c2i = 0; c2i < 16; ++c2i) {
-        float pv[2];
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-          const int c = 2 * c2i + e;
-          if (c < NQ) {
-            const float t = ctrl->tmax[m][c];
-            pv[e] = ex2_approx(sv[c] - (t == -INFINITY ? 0.f : t));
-            v[c] = pv[e];
-          } else {
-            pv[e] = 0.f;
-          }
-        }
-        const uint32_t h0 = __float_as_uint(pv[0]) & 0xffff0000u;
-        const uint32_t h1 = __float_as_uint(pv[1]) & 0xffff0000u;
-        const uint32_t l0 = __float_as_uint(pv[0] - __uint_as_float(h0)) & 0xffff0000u;
-        const uint32_t l1 = __float_as_uint(pv[1] - __uint_as_float(h1)) & 0xffff0000u;
-        hi[c2i] = (h0 >> 16) | h1;
-        lo[c2i] = (l0 >> 16) | l1;
+      for (int c = 0; c < NC; ++c) {
+        const float t = ctrl->tmax[m][c];
+        pv[c] = ex2_approx(sv[c] - (t == -INFINITY ? 0.f : t));
       }
       if (in_pages) {
         uint8_t* prow = smem + LY::kOffP + key * 128;
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
+        for (int j = 0; j < NC / 8; ++j) {
+          uint32_t hi[4], lo[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float p0 = pv[8 * j + 2 * e], p1 = pv[8 * j + 2 * e + 1];
+            const uint32_t h0 = __float_as_uint(p0) & 0xffff0000u;
+            const uint32_t h1 = __float_as_uint(p1) & 0xffff0000u;
+            const uint32_t l0 = __float_as_uint(p0 - __uint_as_float(h0)) & 0xffff0000u;
+            const uint32_t l1 = __float_as_uint(p1 - __uint_as_float(h1)) & 0xffff0000u;
+            hi[e] = (h0 >> 16) | h1;
+            lo[e] = (l0 >> 16) | l1;
+          }
           *reinterpret_cast<uint4*>(prow + ((j ^ (key & 7)) << 4)) =
-              make_uint4(hi[4 * j], hi[4 * j + 1], hi[4 * j + 2], hi[4 * j + 3]);
+              make_uint4(hi[0], hi[1], hi[2], hi[3]);
           *reinterpret_cast<uint4*>(prow + (((j + 4) ^ (key & 7)) << 4)) =
-              make_uint4(lo[4 * j], lo[4 * j + 1], lo[4 * j + 2], lo[4 * j + 3]);
+              make_uint4(lo[0], lo[1], lo[2], lo[3]);
         }
       }
-      const float sm = col_reduce<NQ, false>(v, lane);
-      if (lane < NQ) ctrl->wsum[m][q4][lane] = sm;
+      // column sums over the warp's keys: P in [0, 1] as 24-bit fixed point,
+      // summed exactly by redux (error <= 2^-20 against a tile sum >= 1)
+#pragma unroll
+      for (int c = 0; c < NC; ++c) {
+        const uint32_t u = warp_sum_u32(__float2uint_rn(pv[c] * 16777216.f));
+        if (lane == 0) ctrl->wsum[m][q4][c] = (float)u * (1.f / 16777216.f);
+      }
       // V rows of keys nobody may see are zeroed (after V has landed, or the
       // copy engine would overwrite the zeros); only warps holding such keys
       // (the tail of a sequence, a draft page, a bad page id) wait for V
-      const bool zero = nmin >= NQ && in_pages;
+      const bool zero = nmin >= NC && in_pages;
       if (__any_sync(kFull, zero)) ok = ok && cl_warp_wait(&ctrl->vfull[m], 0);
       if (zero) {
 #pragma unroll
@@ -623,16 +648,14 @@ __global__ void __launch_bounds__(kClThreads, 1)
     }
     // epilogue (group 0: thread = head dim d): tile 0's O^T (P_hi columns +
     // P_lo columns) is read while the other tiles' products run
-    float o0[NQ];
+    float o0[NC];
+#pragma unroll
+    for (int c = 0; c < NC; ++c) o0[c] = 0.f;
     if (m == 0 && ntiles > 0) {
       const bool got = cl_warp_wait(&ctrl->o_full[0], 0);
       ok = ok && got;
       tc_fence_after();
-      float ol[NQ];
-      tmem_ld_cols<NQ>(tmem + lane_off + kClColO, o0);
-      tmem_ld_cols<NQ>(tmem + lane_off + kClColO + 32u, ol);
-#pragma unroll
-      for (int c = 0; c < NQ; ++c) o0[c] = got ? o0[c] + ol[c] : 0.f;
+      if (got) tile_o<NC>(tmem + lane_off + kClColO, min(npg, 8), o0);
     }
     // every tile's statistics are written: the CTA's (max, sum) per column,
     // sent to every CTA of the cluster (all of which are running once the
@@ -640,7 +663,7 @@ __global__ void __launch_bounds__(kClThreads, 1)
     cluster_wait();
     softmax_bar();
     if (warp == 0 && lane < rq) {
-      float M = -INFINITY;
+      float M = -INFINITY;   // (rq <= NC)
       for (int t = 0; t < ntiles; ++t) M = fmaxf(M, ctrl->tmax[t][lane]);
       float L = 0.f;
       for (int t = 0; t < ntiles; ++t) {
@@ -662,21 +685,20 @@ __global__ void __launch_bounds__(kClThreads, 1)
       // the other tiles' O^T, then O^T = sum over tiles of weight x O_t,
       // sent to the CTA that merges dim d (the rows with outputs only)
       const int d = q4 * 32 + lane;
-      float o[NQ];
+      float o[NC];
 #pragma unroll
-      for (int c = 0; c < NQ; ++c) o[c] = ntiles > 0 ? ctrl->tw[0][c] * o0[c] : 0.f;
+      for (int c = 0; c < NC; ++c) o[c] = ntiles > 0 ? ctrl->tw[0][c] * o0[c] : 0.f;
 #pragma unroll 1
       for (int t = 1; t < ntiles; ++t) {
         const bool got = cl_warp_wait(&ctrl->o_full[t], 0);
         ok = ok && got;
         tc_fence_after();
-        float oh[NQ], ol[NQ];
-        tmem_ld_cols<NQ>(tmem + lane_off + kClColO + 64u * t, oh);
-        tmem_ld_cols<NQ>(tmem + lane_off + kClColO + 64u * t + 32u, ol);
-        if (got) {
+        float ot[NC];
 #pragma unroll
-          for (int c = 0; c < NQ; ++c) o[c] = fmaf(ctrl->tw[t][c], oh[c] + ol[c], o[c]);
-        }
+        for (int c = 0; c < NC; ++c) ot[c] = 0.f;
+        if (got) tile_o<NC>(tmem + lane_off + kClColO + 128u * t, min(npg - 8 * t, 8), ot);
+#pragma unroll
+        for (int c = 0; c < NC; ++c) o[c] = fmaf(ctrl->tw[t][c], ot[c], o[c]);
       }
       const int owner = dim_owner(d, S);
       const uint32_t a = map_peer(
@@ -685,7 +707,7 @@ __global__ void __launch_bounds__(kClThreads, 1)
           (uint32_t)owner);
       const uint32_t bar = map_peer(smem_u32(&ctrl->recv_full), (uint32_t)owner);
 #pragma unroll
-      for (int c = 0; c < NQ; c += 4)
+      for (int c = 0; c < NC; c += 4)
         if (c < rq) st_async4(a + c * 4u, o[c], o[c + 1], o[c + 2], o[c + 3], bar);
     }
     if (!ok && lane == 0) raise_err(p.err, SEED_DEVERR_TIMEOUT);
@@ -750,26 +772,32 @@ std::atomic<int> g_cl_clusters[64][3];   // resident clusters of 8, 12, 16 CTAs
 
 constexpr int kClSizes[3] = {8, 12, 16};
 
-template <int NQ, int S>
+template <int NC, int S>
 cudaError_t set_cl_attr() {
-  cudaError_t e = cudaFuncSetAttribute(attn_cl_kernel<128, NQ, S>,
+  cudaError_t e = cudaFuncSetAttribute(attn_cl_kernel<128, NC, S>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)cl_smem_bytes<128, S>());
   if (e != cudaSuccess || S <= 8) return e;
-  return cudaFuncSetAttribute(attn_cl_kernel<128, NQ, S>,
+  return cudaFuncSetAttribute(attn_cl_kernel<128, NC, S>,
                               cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+}
+
+template <int S>
+cudaError_t set_cl_attrs_s() {
+  cudaError_t e;
+  if ((e = set_cl_attr<8, S>()) != cudaSuccess) return e;
+  if ((e = set_cl_attr<16, S>()) != cudaSuccess) return e;
+  if ((e = set_cl_attr<24, S>()) != cudaSuccess) return e;
+  return set_cl_attr<32, S>();
 }
 
 cudaError_t set_cl_attrs(int dev) {
   const uint64_t bit = 1ull << (dev & 63);
   if (g_cl_attr_set.load(std::memory_order_acquire) & bit) return cudaSuccess;
   cudaError_t e;
-  if ((e = set_cl_attr<16, 8>()) != cudaSuccess) return e;
-  if ((e = set_cl_attr<32, 8>()) != cudaSuccess) return e;
-  if ((e = set_cl_attr<16, 12>()) != cudaSuccess) return e;
-  if ((e = set_cl_attr<32, 12>()) != cudaSuccess) return e;
-  if ((e = set_cl_attr<16, 16>()) != cudaSuccess) return e;
-  if ((e = set_cl_attr<32, 16>()) != cudaSuccess) return e;
+  if ((e = set_cl_attrs_s<8>()) != cudaSuccess) return e;
+  if ((e = set_cl_attrs_s<12>()) != cudaSuccess) return e;
+  if ((e = set_cl_attrs_s<16>()) != cudaSuccess) return e;
   g_cl_attr_set.fetch_or(bit, std::memory_order_acq_rel);
   return cudaSuccess;
 }
@@ -816,13 +844,19 @@ int cl_clusters(int i) {
   return n > 0 ? n : 0;
 }
 
-template <int NQ, int S>
-cudaError_t launch_cl_t(const PageMaps& pm, const CUtensorMap& tdk, const CUtensorMap& tdv,
-                        const AttnTcParams& prm, cudaStream_t st) {
+template <int S>
+cudaError_t launch_cl_t(int nc, const PageMaps& pm, const CUtensorMap& tdk,
+                        const CUtensorMap& tdv, const AttnTcParams& prm, cudaStream_t st) {
   cudaLaunchConfig_t cfg;
   cudaLaunchAttribute at[2];
   cl_launch_config(cfg, at, dim3(S, prm.hkv, prm.B), S, cl_smem_bytes<128, S>(), st, true);
-  return cudaLaunchKernelEx(&cfg, attn_cl_kernel<128, NQ, S>, pm, tdk, tdv, prm);
+  switch (nc) {
+    case 8: return cudaLaunchKernelEx(&cfg, attn_cl_kernel<128, 8, S>, pm, tdk, tdv, prm);
+    case 16: return cudaLaunchKernelEx(&cfg, attn_cl_kernel<128, 16, S>, pm, tdk, tdv, prm);
+    case 24: return cudaLaunchKernelEx(&cfg, attn_cl_kernel<128, 24, S>, pm, tdk, tdv, prm);
+    case 32: return cudaLaunchKernelEx(&cfg, attn_cl_kernel<128, 32, S>, pm, tdk, tdv, prm);
+  }
+  return cudaErrorInvalidValue;
 }
 
 }  // namespace
@@ -874,17 +908,11 @@ cudaError_t launch_attn_cl(const AttnTcParams& prm, int cluster, const void* k_c
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if ((e = set_cl_attrs(dev)) != cudaSuccess) return e;
-  const bool n16 = prm.G * prm.W1 <= 16;
+  const int nc = (prm.G * prm.W1 + 7) & ~7;   // query rows rounded up to 8
   switch (cluster) {
-    case 8:
-      return n16 ? launch_cl_t<16, 8>(pm, tdk, tdv, prm, st)
-                 : launch_cl_t<32, 8>(pm, tdk, tdv, prm, st);
-    case 12:
-      return n16 ? launch_cl_t<16, 12>(pm, tdk, tdv, prm, st)
-                 : launch_cl_t<32, 12>(pm, tdk, tdv, prm, st);
-    case 16:
-      return n16 ? launch_cl_t<16, 16>(pm, tdk, tdv, prm, st)
-                 : launch_cl_t<32, 16>(pm, tdk, tdv, prm, st);
+    case 8: return launch_cl_t<8>(nc, pm, tdk, tdv, prm, st);
+    case 12: return launch_cl_t<12>(nc, pm, tdk, tdv, prm, st);
+    case 16: return launch_cl_t<16>(nc, pm, tdk, tdv, prm, st);
   }
   return cudaErrorInvalidValue;
 }

@@ -276,6 +276,16 @@ seed_status_t seed_verify_attn(const seed_cfg_t* cfg, int32_t batch, const void*
                     ws_bytes, err_flag, stream);
 }
 
+int32_t seed_attn_route(const seed_cfg_t* cfg, int32_t batch, int32_t draft, int32_t max_pages) {
+  if (check_cfg(cfg) != SEED_OK || batch < 1 || max_pages < 1) return -1;
+  const int G = cfg->hq / cfg->hkv;
+  const int W1 = draft ? 1 : cfg->kmax + 1;
+  if (!tc_path(cfg->head_dim, G, W1)) return SEED_ROUTE_CUDA_CORE;
+  const int cluster = seedk::attn_cl_route(cfg->head_dim, G, W1, batch, cfg->hkv, max_pages);
+  if (cluster > 0) return cluster;
+  return seedk::attn_kt_supported(cfg->head_dim, G, W1) ? SEED_ROUTE_TC_KEYS : SEED_ROUTE_TC_ROWS;
+}
+
 seed_status_t seed_tree_verify_attn(const seed_cfg_t* cfg, int32_t batch, const void* q,
                                     const int32_t* n_nodes, const uint32_t* anc, seed_kv_t kv,
                                     const int32_t* ctx_lens, float* out, float* lse, void* ws,

@@ -44,7 +44,7 @@ def test_exports_every_declared_function(lib):
 
 
 def test_version_and_strings(lib):
-    assert lib.seed_abi_version() == 3
+    assert lib.seed_abi_version() == 4
     for s in range(7):
         assert len(lib.seed_status_string(s)) > 0
     assert lib.seed_status_string(99) == b"unknown status"
@@ -65,6 +65,20 @@ def test_workspace_bytes_validates_cfg(lib, kw, expect):
     c = cfg(**kw)
     n = lib.seed_workspace_bytes(ctypes.byref(c), 4)
     assert (n > 0) == (expect == OK)
+
+
+def test_attn_route_host_logic(lib):
+    """seed_attn_route rejects bad arguments and picks the CUDA-core and
+    keys-as-rows routes by shape alone (the cluster route needs a GPU)."""
+    def r(c, batch, draft, max_pages):
+        return lib.seed_attn_route(ctypes.byref(c), batch, draft, max_pages)
+    assert r(cfg(head_dim=96), 1, 0, 10) == -1
+    assert r(cfg(), 0, 0, 10) == -1
+    assert r(cfg(), 1, 0, 0) == -1
+    assert r(cfg(head_dim=64, hq=8, hkv=2), 4, 0, 100) == 2            # 4 x 5 rows <= 48
+    assert r(cfg(head_dim=64, hq=8, hkv=2), 4, 1, 100) == 2            # draft: 4 rows
+    assert r(cfg(head_dim=64, hq=64, hkv=8, kmax=8), 4, 0, 100) == 0   # 8 x 9 = 72 rows
+    assert r(cfg(), 64, 0, 4000) == 1                                   # 512 pairs
 
 
 def test_workspace_grows_with_batch(lib):

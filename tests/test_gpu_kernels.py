@@ -86,6 +86,25 @@ CASES = [
 ]
 
 
+@pytest.mark.parametrize("case", [c for c in CASES if c[3] == 128])
+def test_attention_route(S, case):
+    """The cases with few (sequence, KV head) pairs, short page tables and at
+    most 32 query rows run on the cluster kernel; the others on the query-rows
+    tensor-core kernel (G * W1 <= 128 for every head_dim 128 case here)."""
+    B, hq, hkv, D, kmax, max_ctx = case[:6]
+    max_pages = -(-(max_ctx + kmax + 1) // 16) + 1       # as gen.small_case
+    cfg = S.SeedConfig(hq=hq, hkv=hkv, head_dim=D, kmax=kmax)
+    for draft in (True, False):
+        rows = (hq // hkv) * (1 if draft else kmax + 1)
+        route = S.seed_attn_route(cfg, B, draft, max_pages)
+        few = B * hkv <= 7 or (B * hkv <= 8 and max_pages + 2 <= 12 * 19) or \
+            (B * hkv <= 15 and max_pages + 2 <= 8 * 19)
+        if rows <= 32 and few:
+            assert route in (8, 12, 16), (case, draft, route)
+        else:
+            assert route == S.ROUTE_TC_ROWS, (case, draft, route)
+
+
 def make(S, seed, case):
     B, hq, hkv, D, kmax, max_ctx, rnd_pages, ks = case
     c = gen.small_case(seed, B, hq, hkv, D, kmax, max_ctx, rnd_pages, ks)
