@@ -378,10 +378,13 @@ def test_accept_commit_is_bit_exact(S, seed, kmax):
 
 
 @pytest.mark.parametrize("case", [(4, 32, 8, 128, 4, 100, True, 1.0),
-                                  (4, 16, 4, 64, 4, 100, True, 1.0)],
-                         ids=["query_rows_D128", "keys_as_rows_D64"])
+                                  (4, 16, 4, 64, 4, 100, True, 1.0),
+                                  (3, 16, 4, 128, 4, 100, True, 1.0)],
+                         ids=["query_rows_D128", "keys_as_rows_D64", "cluster_D128"])
 def test_device_errors_are_flagged_not_fatal(S, case):
     c = make(S, 6, case)
+    if case[0] == 3:   # 12 pairs and a short page table: the cluster kernel
+        assert S.seed_attn_route(c["cfg"], case[0], False, c["max_pages"]) in (8, 12, 16)
     kv = kv_for(S, c, c["lens"] + c["n_q"])
     B = case[0]
     # negative length / length past capacity

@@ -73,13 +73,15 @@ def test_invalid_cfg_and_empty_batch(lib):
 # B, hq, hkv, D, kmax, max_ctx: long enough contexts that pairs split into
 # several units (the arrival counters in the scratch are used), a D=64 shape
 # on the keys-as-rows kernel (20 query rows per KV head), one on the
-# CUDA-core kernel (72 rows), and the largest kmax.
+# CUDA-core kernel (72 rows), the largest kmax, and 12 pairs with a short
+# page table (the cluster kernel).
 CASES = [
     (6, 32, 8, 128, 4, 3000),
     (5, 32, 8, 128, 8, 1100),
     (4, 16, 16, 128, 16, 700),
     (7, 8, 2, 64, 4, 2500),
     (5, 16, 2, 64, 8, 2500),
+    (3, 16, 4, 128, 4, 1500),
 ]
 
 
