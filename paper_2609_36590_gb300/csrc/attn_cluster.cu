@@ -464,6 +464,7 @@ __global__ void __launch_bounds__(kClThreads, 1)
       }
     }
     const int y = code <= -2 ? kPage * (-2 - code) : 0;
+    const uint64_t kv_pol = policy_evict_first();   // cache pages are read once per call
 #pragma unroll
     for (int kv = 0; kv < 2; ++kv) {
       const uint32_t off = kv == 0 ? LY::kOffK : LY::kOffV;
@@ -474,8 +475,8 @@ __global__ void __launch_bounds__(kClThreads, 1)
           uint64_t* bar = kv == 0 ? &ctrl->kfull[m] : &ctrl->vfull[m];
 #pragma unroll
           for (int h = 0; h < LY::kHalves; ++h)
-            tma_load_4d(smem + off + h * LY::kHalfBytes + (8 * m + lane) * 2048, mp, 64 * h, 0, g,
-                        bpid[m], bar);
+            tma_load_4d_hint(smem + off + h * LY::kHalfBytes + (8 * m + lane) * 2048, mp,
+                             64 * h, 0, g, bpid[m], bar, kv_pol);
         }
       }
       // draft pages: one copy each from the draft scratch

@@ -482,6 +482,7 @@ __global__ void __launch_bounds__(kThreadsKT, 1)
       if (lane == 0) write_merge_plan(p, T, x, x1, b, g, t0, pc, s0);
     }
     int tk = 0, uo = 0;
+    const uint64_t kv_pol = policy_evict_first();   // K is read once per call
     bool ok = true;
     int pid_a = -1, pid_b = -1;
     SeqT sq{};
@@ -558,7 +559,8 @@ __global__ void __launch_bounds__(kThreadsKT, 1)
           const int w = box > 0 ? pid : b, r0 = box > 0 ? 0 : kPage * dpage;
 #pragma unroll
           for (int h = 0; h < GE::kSlabs; ++h)
-            tma_load_4d(kb + h * (kKeys * 128), mk, 64 * h, r0, g, w, &ctrl->k_full[s]);
+            tma_load_4d_hint(kb + h * (kKeys * 128), mk, 64 * h, r0, g, w, &ctrl->k_full[s],
+                             kv_pol);
         }
       }
       if (!ok) break;
@@ -590,6 +592,7 @@ __global__ void __launch_bounds__(kThreadsKT, 1)
   } else if (warp == kWarpProdV) {
     // ------------------------------------------------------------ V copies
     int tv = 0;
+    const uint64_t kv_pol = policy_evict_first();   // V is read once per call
     for (;; ++tv) {
       const int s = tv % GE::kSV, mi = tv % kMetaRing;
       if (!kt_warp_wait(&ctrl->meta_full[mi], (tv / kMetaRing) & 1, ctrl, p.err)) break;
@@ -617,7 +620,8 @@ __global__ void __launch_bounds__(kThreadsKT, 1)
         const int w = box > 0 ? pid : mb, r0 = box > 0 ? 0 : kPage * dpage;
 #pragma unroll
         for (int h = 0; h < GE::kSlabs; ++h)
-          tma_load_4d(vb + h * (kKeys * 128), mv, 64 * h, r0, mg, w, &ctrl->v_full[s]);
+          tma_load_4d_hint(vb + h * (kKeys * 128), mv, 64 * h, r0, mg, w, &ctrl->v_full[s],
+                           kv_pol);
       }
     }
     __syncwarp();

@@ -479,6 +479,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
     // to the descriptor ring, from which the V warp issues the tile's V.
     int tk = 0, uo = 0;
     bool ok = true;
+    const uint64_t kv_pol = policy_evict_first();   // K is read once per call
     // page ids of tiles t and t + 1 of the piece (lanes 0-7, one page each),
     // loaded ahead so that their latency overlaps the copies
     int pid_a = -1, pid_b = -1;
@@ -556,8 +557,8 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
           uint8_t* kb = smem + kOffK + (size_t)s * kKV + lane * 2048u;
           const CUtensorMap* mk = box > 0 ? &pm.k[log2_box(box)] : &tm_dk;
           const int w = box > 0 ? pid : b, r0 = box > 0 ? 0 : kPage * dpage;
-          tma_load_4d(kb, mk, 0, r0, g, w, &ctrl->k_full[s]);
-          tma_load_4d(kb + kHalf, mk, 64, r0, g, w, &ctrl->k_full[s]);
+          tma_load_4d_hint(kb, mk, 0, r0, g, w, &ctrl->k_full[s], kv_pol);
+          tma_load_4d_hint(kb + kHalf, mk, 64, r0, g, w, &ctrl->k_full[s], kv_pol);
         }
       }
       if (!ok) break;
@@ -590,6 +591,7 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
     // ---------------------------------------------------------- V loads
     // V(t) into the V ring once tile t's descriptor is out and PV(t - 3)
     // has freed the slot
+    const uint64_t kv_pol = policy_evict_first();   // V is read once per call
     for (int tv = 0;; ++tv) {
       const int s = tv % kStagesTC, mi = tv % kMetaRing;
       if (!warp_wait(&ctrl->meta_full[mi], (tv / kMetaRing) & 1, ctrl, p.err)) break;
@@ -615,8 +617,8 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
         uint8_t* vb = smem + kOffV + (size_t)s * kKV + lane * 2048u;
         const CUtensorMap* mv = box > 0 ? &pm.v[log2_box(box)] : &tm_dv;
         const int w = box > 0 ? pid : mb, r0 = box > 0 ? 0 : kPage * dpage;
-        tma_load_4d(vb, mv, 0, r0, mg, w, &ctrl->v_full[s]);
-        tma_load_4d(vb + kHalf, mv, 64, r0, mg, w, &ctrl->v_full[s]);
+        tma_load_4d_hint(vb, mv, 0, r0, mg, w, &ctrl->v_full[s], kv_pol);
+        tma_load_4d_hint(vb + kHalf, mv, 64, r0, mg, w, &ctrl->v_full[s], kv_pol);
       }
     }
     __syncwarp();
