@@ -91,10 +91,10 @@ def round_bytes(wl, lens: np.ndarray, k_b: np.ndarray, n_layers: int) -> dict:
 # reported traffic is scaled to the timed launches by their algorithmic bytes,
 # and is null once the kernel's sources differ from the captured ones.
 NCU_TRAFFIC = {
-    (4, "verify"): {"kernel": "attn_tc_kernel", "sources": "72ddf281d832025d",
-                    "dram_bytes": 537897216 + 4000768, "alg_bytes": 537907712},
-    (4, "draft"): {"kernel": "attn_tc_kernel", "sources": "72ddf281d832025d",
-                   "dram_bytes": 537332224 + 3645440, "alg_bytes": 536986112},
+    (4, "verify"): {"kernel": "attn_tc_kernel", "sources": "6c57484b573e618b",
+                    "dram_bytes": 537559296 + 3301888, "alg_bytes": 537907712},
+    (4, "draft"): {"kernel": "attn_tc_kernel", "sources": "6c57484b573e618b",
+                   "dram_bytes": 537240064 + 3094016, "alg_bytes": 536986112},
 }
 
 KERNEL_SOURCES = {
