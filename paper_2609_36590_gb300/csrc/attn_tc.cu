@@ -337,12 +337,19 @@ __global__ void __launch_bounds__(kMergeThreads) attn_merge_kernel(const AttnTcP
   for (int i0 = 0; i0 < nseg; i0 += kMergeBatch) {
     float li[kMergeBatch];
     typename V::T x[kMergeBatch];
+    // only the pieces that exist are loaded: the merge's time is its loads
+    // once the attention kernel has ended, and a batch padded with repeats of
+    // the last piece multiplied them (a pair has 2 or 3 pieces, typically)
 #pragma unroll
     for (int u = 0; u < kMergeBatch; ++u) {
-      const int i = min(i0 + u, nseg - 1);
-      const float* rc = p.part + (size_t)(i == 0 ? slot_lo : 2 * (c_lo + i)) * REC;
-      li[u] = (i0 + u < nseg) ? __ldcg(rc + (size_t)D * Rmax + r) : -INFINITY;
-      x[u] = __ldcg(reinterpret_cast<const typename V::T*>(rc + (size_t)r * D) + lane);
+      li[u] = -INFINITY;
+      x[u] = typename V::T{};
+      if (i0 + u < nseg) {
+        const int i = i0 + u;
+        const float* rc = p.part + (size_t)(i == 0 ? slot_lo : 2 * (c_lo + i)) * REC;
+        li[u] = __ldcg(rc + (size_t)D * Rmax + r);
+        x[u] = __ldcg(reinterpret_cast<const typename V::T*>(rc + (size_t)r * D) + lane);
+      }
     }
 #pragma unroll
     for (int u = 0; u < kMergeBatch; ++u) {
