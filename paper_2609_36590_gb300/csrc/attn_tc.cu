@@ -701,13 +701,18 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
           ++tp;
           did = true;
         }
-        // polls without sleeping (a sleep's wake-up granularity would delay
-        // the next MMA); bounded: a stuck pipeline gives up after ~2^28 polls
+        // polls without sleeping once the first S is out (a sleep's wake-up
+        // granularity would delay the next MMA); before it, nothing can be
+        // ready for microseconds, and a spinning warp would take issue slots
+        // from the producer's range lookup, so it backs off.  Bounded: a stuck
+        // pipeline gives up after ~2^28 polls (~2^22 sleeps before the first S).
         if (did) {
           idle = 0;
-        } else if (++idle > (1u << 28)) {
+        } else if (++idle > (ts == 0 ? (1u << 22) : (1u << 28))) {
           ctrl->abort_flag = 1;
           raise_err(p.err, SEED_DEVERR_TIMEOUT);
+        } else if (ts == 0) {
+          __nanosleep(128);
         }
       }
       // Wake both softmax groups through their S barriers: their next tiles,
@@ -747,7 +752,12 @@ __global__ void attn_tc_kernel(const __grid_constant__ CUtensorMap tm_q,
       const int s = t % kStagesTC;
       // S(t) done implies K(t) landed and tile t's descriptor is written; the
       // MMA thread also completes this phase, without an S, at the end
-      if (!warp_wait_hot(&ctrl->s_full[par], own & 1, ctrl, p.err)) break;
+      // (the first S comes microseconds after the dependency wait: that wait
+      // sleeps between tries, so as not to take issue slots from the
+      // producer's lookup on the same sub-partition)
+      if (!(own == 0 ? warp_wait(&ctrl->s_full[par], 0, ctrl, p.err)
+                     : warp_wait_hot(&ctrl->s_full[par], own & 1, ctrl, p.err)))
+        break;
       if (t >= *reinterpret_cast<volatile int32_t*>(&ctrl->end_tile)) break;
       const TileMeta m = ctrl->meta[t % kMetaRing];
       tc_fence_after();
