@@ -91,10 +91,10 @@ def round_bytes(wl, lens: np.ndarray, k_b: np.ndarray, n_layers: int) -> dict:
 # reported traffic is scaled to the timed launches by their algorithmic bytes,
 # and is null once the kernel's sources differ from the captured ones.
 NCU_TRAFFIC = {
-    (4, "verify"): {"kernel": "attn_tc_kernel", "sources": "6c57484b573e618b",
-                    "dram_bytes": 537559296 + 3301888, "alg_bytes": 537907712},
-    (4, "draft"): {"kernel": "attn_tc_kernel", "sources": "6c57484b573e618b",
-                   "dram_bytes": 537240064 + 3094016, "alg_bytes": 536986112},
+    (4, "verify"): {"kernel": "attn_tc_kernel", "sources": "a9f183f7f0271aeb",
+                    "dram_bytes": 537557760 + 3322112, "alg_bytes": 537907712},
+    (4, "draft"): {"kernel": "attn_tc_kernel", "sources": "a9f183f7f0271aeb",
+                   "dram_bytes": 537235712 + 3060480, "alg_bytes": 536986112},
 }
 
 KERNEL_SOURCES = {
