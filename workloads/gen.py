@@ -14,8 +14,9 @@ Recipe
   ``SeedSequence`` stream keyed by the block's coordinates.  A block can
   therefore be regenerated on its own, which lets the oracle check sampled
   outputs of full-size runs without materialising the whole cache on the host.
-* Key-stress rows (workload 4): each key row (layer, b, h, pos) of the initial
-  context is scaled by 8 with probability ``key_stress``, drawn per block.
+* Key-stress rows (the batch-4, 32k-prefix long-context workload): each key
+  row (layer, b, h, pos) of the initial context is scaled by 8 with
+  probability ``key_stress``, drawn per block.
   Multiplying a bf16 value by 8 is exact.
 * Context lengths, draft lengths, acceptance patterns, token ids and page
   orders each come from their own keyed stream.
